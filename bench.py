@@ -1,0 +1,432 @@
+#!/usr/bin/env python3
+"""Benchmark: fused OPD reverse-KL forward+backward on one GB300.
+
+One step = one call of opd_kl_fwd_bwd (row compaction, gather, fused
+student/teacher LM-head forward with online log-sum-exp, combine, fused
+recompute emitting dz, dH_s and dW_s GEMMs, scatter) over one synthetic packed
+batch of the Qwen3-1.7B-shaped workload (T = 16,384 tokens, d_s = 2048,
+d_t = 4096, V = 151,936, bf16). Metric: supervised response tokens per second.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Inputs stay resident in HBM for `value`; `e2e` repeats the measurement through
+the same C ABI with the per-step inputs copied from pinned host memory and the
+per-token KL copied back every step. W_s + W_t (1.87 GB) exceed L2 (129 MB), so
+every step streams the heads from HBM. `--impl reference` times the float64
+CPU oracle on a bounded row sample of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import shutil
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2609_36608_gb300 import synth  # noqa: E402
+
+METRIC = "response tokens/s and % bf16 tensor peak, fused OPD KL fwd+bwd (1 GB300)"
+UNIT = "response tokens/s"
+DEFAULT_WORKLOAD = "qwen3_1p7b"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+KERNEL_SOURCES = {
+    "fused_logits_fwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+    "fused_logits_bwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+    "gemm_dH": ["paper_2609_36608_gb300/csrc/opd_gemm.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+    "gemm_dW": ["paper_2609_36608_gb300/csrc/opd_gemm.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# --------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) of the benchmarked GPU while the timed region runs."""
+
+    FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+              "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+              "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+
+    def __init__(self, device_index: int):
+        self.rows = []
+        self.proc = None
+        self.thread = None
+        exe = shutil.which("nvidia-smi")
+        if exe is None:
+            return
+        ident = None
+        try:
+            ident = "GPU-" + str(torch.cuda.get_device_properties(device_index).uuid)
+        except Exception:
+            vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+            ident = vis.split(",")[device_index] if vis else str(device_index)
+        self.cmd = [exe, "-i", ident, "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
+                    "-lms", "200"]
+
+    def start(self):
+        if not hasattr(self, "cmd"):
+            return
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == len(self.FIELDS):
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+
+    def summary(self):
+        if not self.rows:
+            return None
+        sm = [float(r[0]) for r in self.rows if re.match(r"^[\d.]+$", r[0])]
+        mx = [float(r[1]) for r in self.rows if re.match(r"^[\d.]+$", r[1])]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[4 + i].lower().startswith("active")})
+        pw = [float(r[2]) for r in self.rows if re.match(r"^[\d.]+$", r[2])]
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows), "power_w_max": max(pw) if pw else None}
+
+
+# ------------------------------------------------------------------ distributed
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def init_dist(world, backend):
+    if world > 1 and not torch.distributed.is_initialized():
+        torch.distributed.init_process_group(backend=backend)
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+# -------------------------------------------------------------------- flops
+
+def step_flops(w, R):
+    executed = R * w.V * (8 * w.d_s + 4 * w.d_t)
+    algorithmic = R * w.V * (6 * w.d_s + 2 * w.d_t)
+    return executed, algorithmic
+
+
+def kernel_flops(name, w, R):
+    if name in ("fused_logits_fwd", "fused_logits_bwd"):
+        return 2.0 * R * w.V * (w.d_s + w.d_t)
+    if name in ("gemm_dH", "gemm_dW"):
+        return 2.0 * R * w.V * w.d_s
+    return None
+
+
+def source_hash(name):
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES.get(name, []):
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(name, workload):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source still matches."""
+    path = os.path.join(ROOT, "profiles", f"{name}_{workload}.txt")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_b = re.search(r"^dram_bytes_per_launch:\s*([\d.eE+]+)", text, re.M)
+    m_h = re.search(r"^source_sha256:\s*([0-9a-f]{64})", text, re.M)
+    if not m_b or not m_h or m_h.group(1) != source_hash(name):
+        return None
+    return float(m_b.group(1))
+
+
+# ---------------------------------------------------------------- CPU oracle
+
+def oracle_rate(w, host, lay, g, rows, threads):
+    import oracle
+    oracle.build()
+    t0 = time.perf_counter()
+    oracle.opd_kl(host["H_s"], host["H_t"], host["W_s"], host["W_t"], lay.mask, g, w.tau, rows=rows,
+                  want_dH=True, want_dW=True, n_threads=threads)
+    dt = time.perf_counter() - t0
+    return len(rows) / dt, dt
+
+
+def host_inputs(x):
+    return {k: synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")}
+
+
+def sample_rows(mask, n, offset=0):
+    sup = np.flatnonzero(mask)
+    if len(sup) == 0:
+        return sup
+    idx = (np.arange(n) * max(1, len(sup) // n) + offset) % len(sup)
+    return sup[np.unique(idx)]
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    w = synth.WORKLOADS[args.workload]
+    lay = synth.layout(w)
+    gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
+    x = synth.hidden_and_heads(w, gen_dev)
+    host = host_inputs(x)
+    del x
+    g = np.where(lay.mask != 0, synth.uniform_weights(w.seed, w.T), 0.0)
+    threads = os.cpu_count() or 1
+    rows_per_step = args.ref_rows
+    import oracle
+    oracle.build()
+    for i in range(args.warmup):
+        oracle_rate(w, host, lay, g, sample_rows(lay.mask, rows_per_step, 7 * i), threads)
+    t0 = time.perf_counter()
+    n = 0
+    for i in range(args.steps):
+        rows = sample_rows(lay.mask, rows_per_step, 13 * i + 1)
+        oracle_rate(w, host, lay, g, rows, threads)
+        n += len(rows)
+    dt = time.perf_counter() - t0
+    value = n / dt
+    sample = (f"{rows_per_step} supervised rows of {w.name} per step (full V={w.V}, d_s={w.d_s}, d_t={w.d_t}): "
+              f"logits, KL, dH_s rows and their dW_s contribution in float64")
+    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * dt / max(args.steps, 1),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+           "data": "synthetic", "config": {"workload": w.name, "T": w.T, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
+                                           "temperature": w.tau},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def run_gpu(args):
+    world, rank, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (the reference arm runs with --impl reference)")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    init_dist(world, "nccl")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+
+    w = synth.WORKLOADS[args.workload]
+    lay = synth.layout(w)
+    R = int(lay.mask.sum())
+    x = synth.hidden_and_heads(w, dev)
+    grad_h = opd_kl.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)
+    mask = torch.from_numpy(lay.mask).to(dev)
+    grad = torch.from_numpy(grad_h).to(dev)
+    dtype = opd_kl.OPD_DTYPE_BF16 if w.dtype == "bf16" else opd_kl.OPD_DTYPE_F32
+    prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
+    ws = opd_kl.allocate_workspace(prob, dev)
+    kl = torch.empty(w.T, device=dev)
+    stats = torch.empty(w.T, 3, device=dev)
+    dH = torch.empty(w.T, w.d_s, device=dev)
+    dW = torch.empty(w.V, w.d_s, device=dev)
+
+    def step(H_s, H_t, m, gr):
+        opd_kl.opd_kl_fwd_bwd(prob, H_s, H_t, x["W_s"], x["W_t"], m, gr, kl, stats, dH, dW, False, ws)
+
+    for _ in range(args.warmup):
+        step(x["H_s"], x["H_t"], mask, grad)
+    torch.cuda.synchronize()
+    if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
+        raise RuntimeError("device status after warm-up is not OK")
+
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    opd_kl.opd_kl_profile_start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    for _ in range(args.steps):
+        step(x["H_s"], x["H_t"], mask, grad)
+    ev1.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    prof = opd_kl.opd_kl_profile_stop()
+    if sampler:
+        sampler.stop()
+    if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
+        raise RuntimeError("device status after the timed region is not OK")
+    ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
+    ms_step = ms / args.steps
+    value = R * args.steps * world / (ms / 1000.0)
+
+    # end to end through the same C ABI: inputs from pinned host memory, KL back every step
+    H_s_h = x["H_s"].cpu().pin_memory()
+    H_t_h = x["H_t"].cpu().pin_memory()
+    mask_h = torch.from_numpy(lay.mask).pin_memory()
+    grad_hp = torch.from_numpy(grad_h).pin_memory()
+    kl_h = torch.empty(w.T, dtype=torch.float32).pin_memory()
+    H_s_d, H_t_d = torch.empty_like(x["H_s"]), torch.empty_like(x["H_t"])
+    mask_d, grad_d = torch.empty_like(mask), torch.empty_like(grad)
+    h2d = (H_s_h.numel() * H_s_h.element_size() + H_t_h.numel() * H_t_h.element_size() + mask_h.numel()
+           + grad_hp.numel() * 4)
+    d2h = kl_h.numel() * 4
+
+    def e2e_step():
+        H_s_d.copy_(H_s_h, non_blocking=True)
+        H_t_d.copy_(H_t_h, non_blocking=True)
+        mask_d.copy_(mask_h, non_blocking=True)
+        grad_d.copy_(grad_hp, non_blocking=True)
+        step(H_s_d, H_t_d, mask_d, grad_d)
+        kl_h.copy_(kl, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+        return float(kl_h[0])
+
+    e2e_step()
+    barrier(world)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = R * args.steps * world / (e2e_ms / 1000.0)
+
+    if rank != 0:
+        torch.distributed.destroy_process_group() if world > 1 else None
+        return 0
+
+    peaks, peak_src = load_peaks()
+    executed, algorithmic = step_flops(w, R)
+    kernels = {}
+    total_k = sum(v[1] for v in prof.values()) or 1.0
+    for name, (n, tot) in sorted(prof.items(), key=lambda kv: -kv[1][1]):
+        kernels[name] = {"launches": n, "ms_per_launch": tot / max(n, 1), "share": tot / total_k}
+    heavy = [k for k in kernels if kernel_flops(k, w, R) is not None]
+    dom = max(heavy, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"]) if heavy else None
+    roofline = None
+    if dom:
+        per_launch = kernel_flops(dom, w, R)
+        achieved = per_launch / (kernels[dom]["ms_per_launch"] / 1000.0) / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        traffic = recorded_traffic(dom, w.name)
+        roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "traffic": traffic,
+                    "peak_source": f"bf16_tflops_sustained of {peak_src}",
+                    "frac_of_burst": achieved / peaks["bf16_tflops"],
+                    "algorithmic_flops_per_launch": per_launch}
+
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        host = host_inputs(x)
+        g = np.where(lay.mask != 0, grad_h.astype(np.float64), 0.0)
+        rows = sample_rows(lay.mask, args.cpu_rows, 3)
+        threads = os.cpu_count() or 1
+        rate, dt = oracle_rate(w, host, lay, g, rows, threads)
+        cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": f"{len(rows)} supervised rows of {w.name}: float64 logits, KL, dH_s rows and their "
+                         f"dW_s contribution ({dt:.1f} s)"}
+
+    clocks = sampler.summary() if sampler else None
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded counter-based generator, packed multi-turn layout with masked observations "
+                "and inserted tokens",
+        "config": {"workload": w.name, "T": w.T, "R": R, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
+                   "temperature": w.tau, "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (W_s + W_t = %.2f GB)" % ((w.d_s + w.d_t) * w.V * 2 / 1e9)},
+        "tflops_executed": executed / (ms_step / 1000.0) / 1e12,
+        "tflops_algorithmic": algorithmic / (ms_step / 1000.0) / 1e12,
+        "pct_bf16_peak_executed": 100.0 * executed / (ms_step / 1000.0) / 1e12 / peaks["bf16_tflops"],
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
+        "clocks": clocks,
+        "kernels": kernels,
+    }
+    print(json.dumps(out), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
+    ap.add_argument("--ref-rows", type=int, default=8, help="rows per step of --impl reference")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        log("note: at least 3 warm-up steps are required for a valid measurement; using 3")
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

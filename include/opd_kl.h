@@ -1,0 +1,149 @@
+/*
+ * opd_kl.h: C ABI of the fused on-policy-distillation reverse-KL step on one
+ * NVIDIA GB300 (sm_103a).
+ *
+ * What is computed (ActFirst-OPD, Section 3, Eq. opd-objective and
+ * Eq. reverse-kl; masking and the frozen teacher from Appendix B.4):
+ *
+ *   for every packed token row i with mask[i] = 1 (a model-generated response
+ *   token; prompts, observations, inserted thinking-budget tokens and padding
+ *   have mask 0):
+ *     z_s = H_s[i,:] W_s^T,  z_t = H_t[i,:] W_t^T         (length V logits)
+ *     u = z / temperature,   log p = u - logsumexp(u)     (student s, teacher t)
+ *     KL_i = sum_v p_s[v] (log p_s[v] - log p_t[v])       reverse KL, student || teacher
+ *   and, given upstream weights g_i = dL/dKL_i,
+ *     dz_i[v] = (g_i / temperature) p_s[v] (log p_s[v] - log p_t[v] - KL_i)
+ *     dH_s[i,:] = dz_i W_s,    dW_s = sum_i dz_i^T H_s[i,:]
+ *   Rows with mask 0 get KL_i = 0 and dH_s[i,:] = 0 and add nothing to dW_s.
+ *   The teacher is frozen: no gradient for H_t or W_t.
+ *
+ * Layouts: every matrix is dense row-major.
+ *   H_s [T, d_s], H_t [T, d_t]   hidden states at the token positions
+ *   W_s [V, d_s], W_t [V, d_t]   LM heads in nn.Linear layout (z = H W^T)
+ *   mask [T] uint8 (nonzero = supervised), kl_out [T] float, stats [T, 3] float
+ *   (lse_s, lse_t, KL per row, natural log; zeros on unsupervised rows),
+ *   grad_kl [T] float, dH_s [T, d_s] float, dW_s [V, d_s] float.
+ *
+ * Element types: OPD_DTYPE_BF16 runs the tcgen05 tensor-core path (bf16 inputs,
+ * fp32 accumulation, fp32 outputs); it needs d_s and d_t multiples of 8 and
+ * 16-byte aligned base addresses. OPD_DTYPE_F32 runs a CUDA-core fp32 path.
+ *
+ * Ownership: the caller owns and allocates every buffer (device memory),
+ * including the workspace; the library allocates nothing, keeps no pointer
+ * after a call returns, and enqueues all work on the given stream without
+ * synchronising it (unless OPD_KL_SYNC_CHECK=1 is set in the environment, which
+ * makes every call synchronise and report device-side errors).
+ *
+ * Errors: every argument is validated on the host before any launch; a bad
+ * argument returns OPD_ERR_INVALID_ARG or OPD_ERR_UNSUPPORTED and launches
+ * nothing. Launch failures return OPD_ERR_CUDA. Device-side failures (a bounded
+ * wait that ran out) set a status word inside the workspace; read it with
+ * opd_kl_get_status. Nothing ever traps the GPU.
+ *
+ * Streams are passed as void* and are cudaStream_t values (NULL = legacy default stream).
+ */
+#ifndef OPD_KL_H
+#define OPD_KL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  OPD_OK = 0,
+  OPD_ERR_INVALID_ARG = 1, /* null pointer, bad size, misaligned buffer, workspace too small */
+  OPD_ERR_UNSUPPORTED = 2, /* valid but not handled (e.g. bf16 with d % 8 != 0) */
+  OPD_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed */
+  OPD_ERR_TIMEOUT = 4,     /* a device-side bounded wait ran out (see opd_kl_get_status) */
+  OPD_ERR_NONFINITE = 5    /* reserved: non-finite inputs are undefined behaviour, not checked */
+} opd_status;
+
+typedef enum { OPD_DTYPE_BF16 = 0, OPD_DTYPE_F32 = 1 } opd_dtype;
+
+/* One problem: T packed token rows, hidden sizes, vocabulary size, element type
+ * of H_s/H_t/W_s/W_t, and the softmax temperature applied to both policies. */
+typedef struct {
+  int64_t T;
+  int64_t d_s;
+  int64_t d_t;
+  int64_t V;
+  int32_t dtype;       /* opd_dtype */
+  float temperature;   /* > 0 */
+} opd_problem;
+
+/* Bytes of device workspace that forward, backward and fwd_bwd need for this
+ * problem (an upper bound: it assumes every row may be supervised). Returns 0
+ * for an invalid problem. The workspace must be 256-byte aligned. Its largest
+ * part is the bf16 dz buffer of T x V elements. */
+size_t opd_kl_workspace_size(const opd_problem* problem);
+
+/* Forward (Eq. reverse-kl): per-token KL and the per-row statistics the backward
+ * needs. kl_out [T] and stats [T, 3] are written for every row (zeros on
+ * unsupervised rows). */
+opd_status opd_kl_forward(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                          const void* W_t, const uint8_t* mask, float* kl_out, float* stats, void* workspace,
+                          size_t workspace_bytes, void* stream);
+
+/* Backward: given stats from opd_kl_forward on the same inputs and grad_kl [T]
+ * (dL/dKL_i; entries on unsupervised rows are ignored), writes dH_s [T, d_s]
+ * (zeros on unsupervised rows) and dW_s [V, d_s]; with accumulate_dW != 0 the
+ * dW_s contribution is added to what dW_s already holds. */
+opd_status opd_kl_backward(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                           const void* W_t, const uint8_t* mask, const float* stats, const float* grad_kl,
+                           float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
+                           void* stream);
+
+/* Forward then backward in one call (row compaction and gathering done once):
+ * writes kl_out, stats, dH_s and dW_s as the two calls above would. */
+opd_status opd_kl_fwd_bwd(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                          const void* W_t, const uint8_t* mask, const float* grad_kl, float* kl_out, float* stats,
+                          float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
+                          void* stream);
+
+/* Host helper (Appendix B.4, Eq. opd-surrogate, seq-mean-token-mean): upstream
+ * weights w_i = dL/dl_i for L = 1/|B| sum_b (sum_j m_bj l_bj) / (sum_j m_bj + eps).
+ * seg_id [T]: response index of row i (>= 0) or negative outside any response;
+ * |B| = number of distinct non-negative ids. w_out [T] host memory; rows with
+ * mask 0 or a negative id get 0. Returns OPD_ERR_INVALID_ARG on null pointers
+ * (with T > 0), T < 0 or eps < 0. */
+opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t* mask, int64_t T, float eps,
+                                           float* w_out);
+
+/* Reads and clears the device status word in the workspace, after
+ * synchronising the stream: OPD_OK, or OPD_ERR_TIMEOUT if a bounded wait in the
+ * last call ran out. */
+opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stream);
+
+/* Self-test of the bounded-wait machinery: launches one kernel that waits on a
+ * barrier nothing completes, with the given limit (nanoseconds, at most 1e9),
+ * then reads the status as opd_kl_get_status does. Returns OPD_ERR_TIMEOUT when
+ * the wait gave up as designed; the CUDA context stays usable. */
+opd_status opd_kl_selftest_timeout(void* workspace, size_t workspace_bytes, uint64_t limit_ns, void* stream);
+
+/* Per-kernel timing of the library's own launches, for roofline accounting.
+ * Between opd_kl_profile_start and opd_kl_profile_stop every kernel the library
+ * launches is bracketed by two CUDA events recorded on the caller's stream (off
+ * by default; when on it adds two event records per launch). stop() waits for
+ * those events, then writes up to `capacity` entries (one per kernel name: launch
+ * count and summed event time in milliseconds) to `out` (host memory), sets
+ * *n_out to the number of distinct kernels, and turns timing off. */
+typedef struct {
+  char name[48];
+  int64_t launches;
+  double total_ms;
+} opd_kernel_time;
+
+opd_status opd_kl_profile_start(void);
+opd_status opd_kl_profile_stop(opd_kernel_time* out, int capacity, int* n_out);
+
+/* Human-readable name of a status code (static storage). */
+const char* opd_status_string(opd_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OPD_KL_H */

@@ -1,0 +1,237 @@
+// Memory-bound steps around the tensor-core kernels:
+//   compaction  mask[T] -> idx[R] (supervised rows in order), pos[T] (rank or -1)
+//               (Appendix B.4: m = 1 on model-generated response tokens only)
+//   gather      H_s, H_t rows -> contiguous [R_pad, d] bf16 buffers, zero rows R..R_pad-1
+//   combine     per-split statistics -> lse_s, lse_t, KL per token (Eq. reverse-kl)
+//   bwd_rowc    per-row constants of dz = (g/tau) p_s (log p_s - log p_t - KL)
+//   zero_rows / scatter_rows   dH_s partial-sum buffer, then back to the T rows
+#include <math_constants.h>
+
+#include "opd_device.cuh"
+#include "opd_internal.h"
+
+namespace opd {
+
+namespace {
+
+constexpr int kCompactThreads = 1024;
+
+// One CTA: each thread counts the mask over a contiguous slice, a block-wide
+// exclusive scan gives each slice its output offset, then the slice is written.
+__global__ void __launch_bounds__(kCompactThreads)
+    k_compact(const uint8_t* __restrict__ mask, int32_t T, int32_t* __restrict__ idx, int32_t* __restrict__ pos,
+              Ctrl* ctrl) {
+  __shared__ int32_t warp_tot[32];
+  const int tid = threadIdx.x;
+  if (tid == 0) ctrl->status = 0u;
+  const int per = (T + kCompactThreads - 1) / kCompactThreads;
+  const int lo = min(T, tid * per);
+  const int hi = min(T, lo + per);
+  int cnt = 0;
+  for (int i = lo; i < hi; ++i) cnt += mask[i] != 0;
+  // inclusive warp scan, then scan of warp totals
+  const int lane = tid & 31, w = tid >> 5;
+  int x = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tot[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    int t = warp_tot[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, t, o);
+      if (lane >= o) t += y;
+    }
+    warp_tot[lane] = t;  // inclusive totals
+  }
+  __syncthreads();
+  int off = x - cnt + (w > 0 ? warp_tot[w - 1] : 0);
+  for (int i = lo; i < hi; ++i) {
+    if (mask[i] != 0) {
+      idx[off] = i;
+      pos[i] = off;
+      ++off;
+    } else {
+      pos[i] = -1;
+    }
+  }
+  if (tid == kCompactThreads - 1) {
+    ctrl->R = warp_tot[31];
+    ctrl->n_vsplit = 0;
+  }
+}
+
+// Row gather in 16-byte vectors; rows in [R, R_pad) become zero.
+__global__ void k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict__ Ht, int32_t vs, int32_t vt,
+                          const int32_t* __restrict__ idx, const Ctrl* __restrict__ ctrl, uint4* __restrict__ Hs_g,
+                          uint4* __restrict__ Ht_g) {
+  const int R = ctrl->R;
+  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  const int per_row = vs + vt;
+  const long total = (long)R_pad * per_row;
+  for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x) {
+    const int r = (int)(e / per_row);
+    const int v = (int)(e - (long)r * per_row);
+    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    if (v < vs) {
+      if (r < R) val = Hs[(long)idx[r] * vs + v];
+      Hs_g[(long)r * vs + v] = val;
+    } else {
+      const int v2 = v - vs;
+      if (r < R) val = Ht[(long)idx[r] * vt + v2];
+      Ht_g[(long)r * vt + v2] = val;
+    }
+  }
+}
+
+// Merge the base-2 statistics of every vocabulary split of one row:
+//   M = max_j m_j,  S = sum_j S_j 2^(m_j - M),  A likewise
+// then  lse = (M + log2 S) ln 2,  KL = (A_s / S_s) ln 2 - lse_s + lse_t.
+__global__ void k_combine(const float* __restrict__ part, const int32_t* __restrict__ pos,
+                          const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
+                          float* __restrict__ stats) {
+  const int n_vs = ctrl->n_vsplit;
+  const size_t plane = (size_t)T_pad;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+    const int r = pos[i];
+    float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
+    if (r >= 0 && n_vs > 0) {
+      float Ms = -CUDART_INF_F, Mt = -CUDART_INF_F;
+      for (int j = 0; j < n_vs; ++j) {
+        const float* b = part + (size_t)j * 5 * plane + r;
+        Ms = fmaxf(Ms, b[0]);
+        Mt = fmaxf(Mt, b[3 * plane]);
+      }
+      float Ss = 0.f, As = 0.f, St = 0.f;
+      for (int j = 0; j < n_vs; ++j) {
+        const float* b = part + (size_t)j * 5 * plane + r;
+        const float fs = exp2f(b[0] - Ms);
+        Ss = fmaf(b[plane], fs, Ss);
+        As = fmaf(b[2 * plane], fs, As);
+        St = fmaf(b[4 * plane], exp2f(b[3 * plane] - Mt), St);
+      }
+      const float ln2 = 0.69314718055994531f;
+      lse_s = (Ms + log2f(Ss)) * ln2;
+      lse_t = (Mt + log2f(St)) * ln2;
+      kl = (As / Ss) * ln2 - lse_s + lse_t;
+    }
+    kl_out[i] = kl;
+    stats[3 * (size_t)i + 0] = lse_s;
+    stats[3 * (size_t)i + 1] = lse_t;
+    stats[3 * (size_t)i + 2] = kl;
+  }
+}
+
+__global__ void k_bwd_rowc(const float* __restrict__ stats, const float* __restrict__ grad_kl,
+                           const int32_t* __restrict__ idx, const Ctrl* __restrict__ ctrl, int32_t T_pad, float tau,
+                           float4* __restrict__ rowc) {
+  const int R = ctrl->R;
+  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R_pad; r += gridDim.x * blockDim.x) {
+    float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (r < R) {
+      const int i = idx[r];
+      const float lse_s = stats[3 * (size_t)i + 0];
+      const float lse_t = stats[3 * (size_t)i + 1];
+      const float kl = stats[3 * (size_t)i + 2];
+      c.x = lse_s * 1.4426950408889634f;
+      c.y = lse_s - lse_t + kl;
+      c.z = grad_kl[i] / tau;
+    }
+    rowc[r] = c;
+  }
+}
+
+__global__ void k_zero_rows(float4* __restrict__ buf, int32_t vec_per_row, const Ctrl* __restrict__ ctrl) {
+  const int R = ctrl->R;
+  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  const long total = (long)R_pad * vec_per_row;
+  for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x)
+    buf[e] = make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+__global__ void k_scatter_rows(const float4* __restrict__ src, int32_t vec_per_row, const int32_t* __restrict__ pos,
+                               int32_t T, float4* __restrict__ dst) {
+  const long total = (long)T * vec_per_row;
+  for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x) {
+    const int i = (int)(e / vec_per_row);
+    const int v = (int)(e - (long)i * vec_per_row);
+    const int r = pos[i];
+    dst[e] = r >= 0 ? src[(long)r * vec_per_row + v] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+// Waits on an mbarrier that nothing will ever complete, to exercise the bounded
+// wait: it must give up after limit_ns, flag kDevTimeout and return.
+__global__ void k_selftest_timeout(Ctrl* ctrl, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    ctrl->status = 0u;
+    mbar_wait(&bar, 0u, &ctrl->status, limit_ns);
+  }
+}
+
+int grid_for(long work, int n_sm, int threads) {
+  long g = (work + threads - 1) / threads;
+  const long cap = (long)n_sm * 8;
+  if (g > cap) g = cap;
+  return (int)(g < 1 ? 1 : g);
+}
+
+}  // namespace
+
+cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t* pos, Ctrl* ctrl,
+                           cudaStream_t s) {
+  k_compact<<<1, kCompactThreads, 0, s>>>(mask, T, idx, pos, ctrl);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, int32_t d_t, const int32_t* idx,
+                               const Ctrl* ctrl, void* Hs_g, void* Ht_g, int32_t T_pad, int n_sm, cudaStream_t s) {
+  const int vs = d_s / 8, vt = d_t / 8;  // 8 bf16 per 16-byte vector
+  k_gather2<<<grid_for((long)T_pad * (vs + vt), n_sm, 256), 256, 0, s>>>(
+      static_cast<const uint4*>(H_s), static_cast<const uint4*>(H_t), vs, vt, idx, ctrl,
+      static_cast<uint4*>(Hs_g), static_cast<uint4*>(Ht_g));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
+                           float* kl_out, float* stats, int n_sm, cudaStream_t s) {
+  k_combine<<<grid_for(T, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_rowc(const float* stats, const float* grad_kl, const int32_t* idx, const Ctrl* ctrl,
+                            int32_t T_pad, float tau, float4* rowc, cudaStream_t s) {
+  k_bwd_rowc<<<(T_pad + 255) / 256, 256, 0, s>>>(stats, grad_kl, idx, ctrl, T_pad, tau, rowc);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t T_pad, int n_sm, cudaStream_t s) {
+  k_zero_rows<<<grid_for((long)T_pad * cols / 4, n_sm, 256), 256, 0, s>>>(reinterpret_cast<float4*>(buf), cols / 4,
+                                                                           ctrl);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_rows(const float* src_g, int32_t cols, const int32_t* pos, int32_t T, float* dst,
+                                int n_sm, cudaStream_t s) {
+  k_scatter_rows<<<grid_for((long)T * cols / 4, n_sm, 256), 256, 0, s>>>(
+      reinterpret_cast<const float4*>(src_g), cols / 4, pos, T, reinterpret_cast<float4*>(dst));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_selftest_timeout(Ctrl* ctrl, uint64_t limit_ns, cudaStream_t s) {
+  k_selftest_timeout<<<1, 32, 0, s>>>(ctrl, limit_ns);
+  return cudaGetLastError();
+}
+
+}  // namespace opd

@@ -1,0 +1,297 @@
+// Gradient GEMMs of the OPD reverse-KL step on tcgen05 (bf16 in, fp32 out):
+//
+//   dH_s = dZ W_s      M = supervised rows, N = d_s, K = V   (A K-major, B MN-major)
+//   dW_s = dZ^T H_s    M = V, N = d_s, K = supervised rows   (A and B MN-major)
+//
+// dZ is the bf16 gradient of the weighted per-token KL with respect to the
+// student logits, written by the fused backward kernel. The teacher is frozen
+// (Appendix B.4), so there is no teacher gradient.
+//
+// Tiles: 128 x 256 fp32 accumulators in TMEM (two buffers = 512 columns), 64-deep
+// K blocks staged by TMA with 128-byte swizzle, one thread issuing MMAs, four
+// epilogue warps draining TMEM through swizzled shared memory into TMA stores
+// (or TMA reduce-adds, for split-K partial sums and for accumulating into dW_s).
+#include "opd_device.cuh"
+#include "opd_internal.h"
+
+namespace opd {
+
+namespace {
+
+constexpr int kBN = kGemmBN;
+constexpr int kStages = 4;
+constexpr uint32_t kABytes = kRowTile * kKBlock * 2;  // 16 KB
+constexpr uint32_t kBBytes = kBN * kKBlock * 2;       // 32 KB
+constexpr uint32_t kStageBytes = kABytes + kBBytes;
+constexpr uint32_t kChunkBytes = 32 * 32 * 4;         // one 32x32 fp32 staging box
+constexpr uint32_t kStagingPerWarp = 2 * kChunkBytes;
+constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 4 * kStagingPerWarp + 256;
+static_assert(kSmem <= 232448, "shared memory budget");
+
+struct GemmSchedule {
+  int n_mt, n_nt, nkb, n_ks, n_units;
+
+  __device__ void init(int M, int N, int K, int grid, int max_ks) {
+    n_mt = (M + kRowTile - 1) / kRowTile;
+    n_nt = (N + kBN - 1) / kBN;
+    nkb = (K + kKBlock - 1) / kKBlock;
+    n_ks = 1;
+    if (max_ks > 1 && n_mt > 0 && nkb > 1) {
+      long best = -1;
+      const int lim = max_ks < nkb ? max_ks : nkb;
+      for (int s = 1; s <= lim; ++s) {
+        const long waves = ((long)n_mt * n_nt * s + grid - 1) / grid;
+        const long cost = waves * ((nkb + s - 1) / s);
+        if (best < 0 || cost < best) {
+          best = cost;
+          n_ks = s;
+        }
+      }
+    }
+    n_units = n_mt * n_nt * n_ks;
+  }
+
+  __device__ void unit(int u, int& mt, int& nt, int& kb0, int& kb1) const {
+    nt = u % n_nt;
+    const int r = u / n_nt;
+    mt = r % n_mt;
+    const int ks = r / n_mt;
+    kb0 = (int)(((long)ks * nkb) / n_ks);
+    kb1 = (int)(((long)(ks + 1) * nkb) / n_ks);
+  }
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+__device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  const uint32_t addr = smem_u32(bar);
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0; !mbar_try_wait(addr, parity); ++it) {
+    if ((it & 63u) == 63u && (globaltimer_ns() - t0 > limit_ns || it >= (1u << 28))) return;
+  }
+}
+
+template <bool A_MN, bool B_MN>
+__global__ void __launch_bounds__(192, 1)
+    k_umma_gemm(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
+                const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  uint8_t* stage_base = smem;
+  uint8_t* staging = smem + kStages * kStageBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(staging + 4 * kStagingPerWarp);
+  uint64_t* empty = full + kStages;
+  uint64_t* acc_full = empty + kStages;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* mma_done = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  uint32_t* status = &p.ctrl->status;
+  const uint64_t lim = p.wait_limit_ns;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);
+    }
+    mbar_init(mma_done, 1);
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tm_a);
+    prefetch_tmap(&tm_b);
+    prefetch_tmap(&tm_c);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int R = p.ctrl->R;
+  const int M = p.m_is_R ? R : p.M;
+  const int K = p.k_is_R ? R : p.K;
+  GemmSchedule sch;
+  sch.init(M, p.N, K, gridDim.x, p.max_ksplit);
+
+  if (warp == 0) {
+    if (lane == 0) {
+      uint32_t stage = 0, phase = 0;
+      bool ok = true, any = false;
+      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x) {
+        int mt, nt, kb0, kb1;
+        sch.unit(u, mt, nt, kb0, kb1);
+        const int m0 = mt * kRowTile, n0 = nt * kBN;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, status, lim)) {
+            ok = false;
+            break;
+          }
+          uint8_t* sa = stage_base + stage * kStageBytes;
+          uint8_t* sb = sa + kABytes;
+          const int k0 = kb * kKBlock;
+          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          if (A_MN) {
+            tma_load_2d(sa, &tm_a, &full[stage], m0, k0);
+            tma_load_2d(sa + 8192, &tm_a, &full[stage], m0 + 64, k0);
+          } else {
+            tma_load_2d(sa, &tm_a, &full[stage], k0, m0);
+          }
+          if (B_MN) {
+#pragma unroll
+            for (int i = 0; i < kBN / 64; ++i) tma_load_2d(sb + 8192 * i, &tm_b, &full[stage], n0 + 64 * i, k0);
+          } else {
+            tma_load_2d(sb, &tm_b, &full[stage], k0, n0);
+          }
+          any = true;
+          if (++stage == (uint32_t)kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok && any) {
+        for (int s = 0; s < kStages; ++s) {
+          const uint32_t par = ((uint32_t)s < stage) ? phase : (phase ^ 1u);
+          mbar_wait_drain(&full[s], par, lim);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kRowTile, kBN, A_MN, B_MN);
+      uint32_t stage = 0, phase = 0;
+      int lt = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x, ++lt) {
+        int mt, nt, kb0, kb1;
+        sch.unit(u, mt, nt, kb0, kb1);
+        const int buf = lt & 1;
+        const uint32_t acc_par = (uint32_t)(lt >> 1) & 1u;
+        if (!mbar_wait(&acc_empty[buf], acc_par ^ 1u, status, lim)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(buf * kBN);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, status, lim)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(stage_base + stage * kStageBytes);
+          const uint32_t sb = sa + kABytes;
+#pragma unroll
+          for (int k = 0; k < kKBlock / 16; ++k) {
+            // K-major: the 16-wide K slice starts 32 bytes further along each 128-byte row.
+            // MN-major: it starts 16 rows (2048 bytes) further down; 64-wide MN blocks are 8 KB apart.
+            const uint64_t ad = A_MN ? sdesc_sw128(sa + k * 2048, 8192, 1024) : sdesc_sw128(sa + k * 32, 16, 1024);
+            const uint64_t bd = B_MN ? sdesc_sw128(sb + k * 2048, 8192, 1024) : sdesc_sw128(sb + k * 32, 16, 1024);
+            umma_bf16(d_tmem, ad, bd, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == (uint32_t)kStages) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok) umma_commit(&acc_full[buf]);
+      }
+      umma_commit(mma_done);
+      mbar_wait_drain(mma_done, 0, lim);
+    }
+  } else {
+    const int q = warp & 3;
+    const uint32_t t_lane = (uint32_t)(q * 32) << 16;
+    uint8_t* stg = staging + q * kStagingPerWarp;
+    int lt = 0;
+    int nchunk = 0;
+    for (int u = blockIdx.x; u < sch.n_units; u += gridDim.x, ++lt) {
+      int mt, nt, kb0, kb1;
+      sch.unit(u, mt, nt, kb0, kb1);
+      const int buf = lt & 1;
+      const uint32_t acc_par = (uint32_t)(lt >> 1) & 1u;
+      // warp-uniform outcome: the TMEM loads below are .sync.aligned
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[buf], acc_par, status, lim))) break;
+      tc_fence_after();
+      const bool empty_k = kb1 <= kb0;
+      const int m0 = mt * kRowTile + q * 32, n0 = nt * kBN;
+      if (!(empty_k && p.reduce)) {
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+          if (n0 + c * 32 >= p.N) break;
+          uint32_t r[32];
+          if (!empty_k) {
+            tmem_ld32(tmem_base + t_lane + (uint32_t)(buf * kBN + c * 32), r);
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) r[j] = 0u;
+          }
+          uint8_t* box = stg + (nchunk & 1) * kChunkBytes;
+          if (lane == 0) bulk_wait_read<1>();
+          __syncwarp();
+          const uint32_t bx = smem_u32(box);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            st_shared_v4(bx + sw128_offset((uint32_t)lane, (uint32_t)j), r[4 * j], r[4 * j + 1], r[4 * j + 2],
+                         r[4 * j + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            if (p.reduce)
+              tma_reduce_add_2d(&tm_c, box, n0 + c * 32, m0);
+            else
+              tma_store_2d(&tm_c, box, n0 + c * 32, m0);
+            bulk_commit();
+          }
+          ++nchunk;
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+    }
+    if (lane == 0) bulk_wait_all<0>();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+template <bool A_MN, bool B_MN>
+cudaError_t launch_impl(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const GemmParams& p,
+                        int grid, cudaStream_t s) {
+  auto kern = k_umma_gemm<A_MN, B_MN>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  if (e != cudaSuccess) return e;
+  kern<<<grid, 192, kSmem, s>>>(a, b, c, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                        const GemmParams& p, int grid, cudaStream_t s) {
+  if (!a_mn && !b_mn) return launch_impl<false, false>(a, b, c, p, grid, s);
+  if (!a_mn && b_mn) return launch_impl<false, true>(a, b, c, p, grid, s);
+  if (a_mn && !b_mn) return launch_impl<true, false>(a, b, c, p, grid, s);
+  return launch_impl<true, true>(a, b, c, p, grid, s);
+}
+
+}  // namespace opd

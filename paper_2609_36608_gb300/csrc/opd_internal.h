@@ -1,0 +1,77 @@
+// Internal interface between the C-ABI layer (opd_api.cu) and the kernel
+// translation units. Not installed; not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace opd {
+
+struct Ctrl;
+
+// Tile geometry shared by host and device code.
+constexpr int kRowTile = 128;   // token rows per MMA tile (TMEM lanes)
+constexpr int kKBlock = 64;     // bf16 elements per 128-byte swizzled row
+constexpr int kMaxVSplit = 64;  // vocabulary splits of the forward statistics
+constexpr int kMaxKSplit = 16;  // K splits of the dH_s GEMM
+constexpr int kFusedBN = 128;   // vocabulary columns per fused tile
+constexpr int kGemmBN = 256;    // output columns per gradient-GEMM tile
+
+struct FusedParams {
+  Ctrl* ctrl;
+  int32_t V, d_s, d_t;
+  int32_t T_pad;        // rows of the gathered buffers (multiple of kRowTile)
+  int32_t group_rows;   // row tiles walked together (L2 raster group)
+  float k2;             // log2(e) / tau
+  float inv_tau;
+  uint64_t wait_limit_ns;
+  float* partials;      // forward: [kMaxVSplit][5][T_pad]
+  const float4* rowc;   // backward: [T_pad] = (lse_s log2 e, lse_s - lse_t + KL, g / tau, 0)
+};
+
+struct GemmParams {
+  Ctrl* ctrl;
+  int32_t M, N, K;      // sizes; M or K is replaced by the supervised row count when flagged
+  int32_t m_is_R, k_is_R;
+  int32_t max_ksplit;   // 1 = whole K per tile
+  int32_t reduce;       // 1 = TMA reduce-add into C, 0 = TMA store
+  uint64_t wait_limit_ns;
+};
+
+// aux kernels (opd_aux.cu)
+cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t* pos, Ctrl* ctrl,
+                           cudaStream_t s);
+cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, int32_t d_t, const int32_t* idx,
+                               const Ctrl* ctrl, void* Hs_g, void* Ht_g, int32_t T_pad, int n_sm, cudaStream_t s);
+cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
+                           float* kl_out, float* stats, int n_sm, cudaStream_t s);
+cudaError_t launch_bwd_rowc(const float* stats, const float* grad_kl, const int32_t* idx, const Ctrl* ctrl,
+                            int32_t T_pad, float tau, float4* rowc, cudaStream_t s);
+cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t T_pad, int n_sm, cudaStream_t s);
+cudaError_t launch_scatter_rows(const float* src_g, int32_t cols, const int32_t* pos, int32_t T, float* dst,
+                                int n_sm, cudaStream_t s);
+cudaError_t launch_selftest_timeout(Ctrl* ctrl, uint64_t limit_ns, cudaStream_t s);
+
+// fp32 CUDA-core path (opd_simt.cu)
+cudaError_t launch_simt_forward(const float* H_s, const float* H_t, const float* W_s, const float* W_t,
+                                int32_t T, int32_t d_s, int32_t d_t, int32_t V, float tau, const int32_t* idx,
+                                const int32_t* pos, const Ctrl* ctrl, float* kl_out, float* stats,
+                                cudaStream_t s);
+cudaError_t launch_simt_backward(const float* H_s, const float* H_t, const float* W_s, const float* W_t,
+                                 int32_t T, int32_t d_s, int32_t d_t, int32_t V, float tau, const int32_t* idx,
+                                 const int32_t* pos, const Ctrl* ctrl, const float* stats, const float* grad_kl,
+                                 float* dZ, float* dH_s, float* dW_s, int accumulate_dW, cudaStream_t s);
+
+// tcgen05 kernels (opd_fused.cu, opd_gemm.cu)
+cudaError_t launch_fused_forward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
+                                 const CUtensorMap& wt, const FusedParams& p, int grid, cudaStream_t s);
+cudaError_t launch_fused_backward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
+                                  const CUtensorMap& wt, const CUtensorMap& dz_store, const FusedParams& p,
+                                  int grid, cudaStream_t s);
+// C = A * B^T with A [M, K] and B [N, K] given through tensor maps; a_mn / b_mn select
+// MN-major operand tiles (the operand's contiguous dimension is M or N, not K).
+cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                        const GemmParams& p, int grid, cudaStream_t s);
+
+}  // namespace opd

@@ -1,0 +1,176 @@
+"""Python binding of the C ABI in include/opd_kl.h (ctypes, argument marshalling only).
+
+Every function has the C entry point's name and forwards to it: all of the
+computation runs in the CUDA library libopdkl.so. PyTorch supplies device
+memory and streams. There is no fallback: importing this module fails loudly
+when the library has not been built (``python -m paper_2609_36608_gb300.build``).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+OPD_OK = 0
+OPD_ERR_INVALID_ARG = 1
+OPD_ERR_UNSUPPORTED = 2
+OPD_ERR_CUDA = 3
+OPD_ERR_TIMEOUT = 4
+OPD_ERR_NONFINITE = 5
+
+OPD_DTYPE_BF16 = 0
+OPD_DTYPE_F32 = 1
+
+
+class opd_problem(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int64), ("d_s", ctypes.c_int64), ("d_t", ctypes.c_int64), ("V", ctypes.c_int64),
+                ("dtype", ctypes.c_int32), ("temperature", ctypes.c_float)]
+
+
+class opd_kernel_time(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int64), ("total_ms", ctypes.c_double)]
+
+
+class OpdError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {opd_status_string(status)} ({status})")
+        self.status = status
+
+
+def _load() -> ctypes.CDLL:
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError(f"libopdkl.so is not built ({path}); run python -m paper_2609_36608_gb300.build")
+    lib = ctypes.CDLL(path)
+    P = ctypes.POINTER(opd_problem)
+    vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t
+    sig = {
+        "opd_kl_workspace_size": (sz, [P]),
+        "opd_kl_forward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
+        "opd_kl_backward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, sz, vp]),
+        "opd_kl_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, sz, vp]),
+        "opd_seq_mean_token_mean_weights": (i32, [vp, vp, i64, ctypes.c_float, vp]),
+        "opd_kl_get_status": (i32, [vp, sz, vp]),
+        "opd_kl_selftest_timeout": (i32, [vp, sz, ctypes.c_uint64, vp]),
+        "opd_status_string": (ctypes.c_char_p, [i32]),
+        "opd_kl_profile_start": (i32, []),
+        "opd_kl_profile_stop": (i32, [ctypes.POINTER(opd_kernel_time), i32, ctypes.POINTER(i32)]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+_lib = _load()
+LIBRARY_PATH = _build.LIB
+
+
+def opd_status_string(status: int) -> str:
+    return _lib.opd_status_string(int(status)).decode()
+
+
+def make_problem(T: int, d_s: int, d_t: int, V: int, dtype: int = OPD_DTYPE_BF16,
+                 temperature: float = 1.0) -> opd_problem:
+    return opd_problem(int(T), int(d_s), int(d_t), int(V), int(dtype), float(temperature))
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError("device buffers must be CUDA tensors")
+    if not t.is_contiguous():
+        raise ValueError("buffers must be contiguous")
+    return ctypes.c_void_p(t.data_ptr()) if t.numel() > 0 else None
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, torch.cuda.Stream):
+        stream = stream.cuda_stream
+    return ctypes.c_void_p(int(stream))
+
+
+def _check(status: int, what: str) -> None:
+    if status != OPD_OK:
+        raise OpdError(status, what)
+
+
+def opd_kl_workspace_size(problem: opd_problem) -> int:
+    return int(_lib.opd_kl_workspace_size(ctypes.byref(problem)))
+
+
+def allocate_workspace(problem: opd_problem, device="cuda") -> torch.Tensor:
+    n = opd_kl_workspace_size(problem)
+    if n == 0:
+        raise ValueError("invalid problem")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def opd_kl_forward(problem, H_s, H_t, W_s, W_t, mask, kl_out, stats, workspace, stream=None) -> None:
+    _check(_lib.opd_kl_forward(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
+                               _ptr(kl_out), _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_kl_forward")
+
+
+def opd_kl_backward(problem, H_s, H_t, W_s, W_t, mask, stats, grad_kl, dH_s, dW_s, accumulate_dW: bool,
+                    workspace, stream=None) -> None:
+    _check(_lib.opd_kl_backward(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
+                                _ptr(stats), _ptr(grad_kl), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
+                                _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_kl_backward")
+
+
+def opd_kl_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, grad_kl, kl_out, stats, dH_s, dW_s, accumulate_dW: bool,
+                   workspace, stream=None) -> None:
+    _check(_lib.opd_kl_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
+                               _ptr(grad_kl), _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s),
+                               int(bool(accumulate_dW)), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_kl_fwd_bwd")
+
+
+def opd_seq_mean_token_mean_weights(seg_id, mask, eps: float = 1e-8) -> np.ndarray:
+    s = np.ascontiguousarray(seg_id, dtype=np.int32)
+    m = np.ascontiguousarray(np.asarray(mask) != 0, dtype=np.uint8)
+    w = np.zeros(s.shape[0], dtype=np.float32)
+    _check(_lib.opd_seq_mean_token_mean_weights(s.ctypes.data_as(ctypes.c_void_p), m.ctypes.data_as(ctypes.c_void_p),
+                                                s.shape[0], float(eps), w.ctypes.data_as(ctypes.c_void_p)),
+           "opd_seq_mean_token_mean_weights")
+    return w
+
+
+def opd_kl_get_status(workspace, stream=None) -> int:
+    return int(_lib.opd_kl_get_status(_ptr(workspace), workspace.numel(), _stream(stream)))
+
+
+def opd_kl_selftest_timeout(workspace, limit_ns: int, stream=None) -> int:
+    return int(_lib.opd_kl_selftest_timeout(_ptr(workspace), workspace.numel(), int(limit_ns), _stream(stream)))
+
+
+def opd_kl_profile_start() -> None:
+    _check(_lib.opd_kl_profile_start(), "opd_kl_profile_start")
+
+
+def opd_kl_profile_stop() -> dict:
+    """{kernel name: (launches, total event milliseconds)} since opd_kl_profile_start."""
+    cap = 64
+    buf = (opd_kernel_time * cap)()
+    n = ctypes.c_int(0)
+    _check(_lib.opd_kl_profile_stop(buf, cap, ctypes.byref(n)), "opd_kl_profile_stop")
+    return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].total_ms)) for i in range(min(n.value, cap))}
+
+
+def call_raw(name: str, *args) -> int:
+    """Call an entry point with raw ctypes arguments (argument-validation tests)."""
+    return int(getattr(_lib, name)(*args))

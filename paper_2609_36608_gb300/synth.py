@@ -203,17 +203,17 @@ def _tiny_layout(T: int, alt: bool) -> Layout:
 
 
 def _packed_layout(w: Workload) -> Layout:
-    """n_traj trajectories of traj_len tokens: observation spans U[20,60] (masked)
+    """T tokens in trajectories of traj_len tokens: observation spans U[20,60] (masked)
     alternate with response spans U[40,90] (supervised); ~5% of responses carry a
     20-token masked inserted span (thinking-budget continuation text)."""
     d = Draws(w.seed, STREAM_LAYOUT)
-    T = w.n_traj * w.traj_len
+    T = w.T
     mask = np.zeros(T, np.uint8)
     seg = np.full(T, -1, np.int32)
     spans = []
     rid = 0
-    for b in range(w.n_traj):
-        pos, end = b * w.traj_len, (b + 1) * w.traj_len
+    for b in range((T + w.traj_len - 1) // w.traj_len):
+        pos, end = b * w.traj_len, min(T, (b + 1) * w.traj_len)
         while pos < end:
             n_obs = min(d.randint(20, 60), end - pos)
             spans.append(("obs", pos, n_obs))

@@ -1,0 +1,90 @@
+"""Host-side checks of the C ABI that need no GPU: the library loads, exports
+every entry point include/opd_kl.h declares, validates arguments before any
+CUDA call, sizes the workspace, and its seq-mean-token-mean helper agrees with
+the oracle (Appendix B.4, Eq. opd-surrogate)."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+    return opd_kl
+
+
+def _declared_functions():
+    text = open(os.path.join(ROOT, "include", "opd_kl.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s*(opd_[a-z0-9_]+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared_functions()
+    assert "opd_kl_forward" in names and "opd_kl_backward" in names and len(names) >= 8
+    so = ctypes.CDLL(lib.LIBRARY_PATH)
+    for n in names:
+        assert hasattr(so, n), n
+
+
+def test_status_strings(lib):
+    assert lib.opd_status_string(0) == "OPD_OK"
+    assert lib.opd_status_string(4) == "OPD_ERR_TIMEOUT"
+    assert lib.opd_status_string(99) == "OPD_ERR_UNKNOWN"
+
+
+def test_workspace_size(lib):
+    p = lib.make_problem(16384, 2048, 4096, 151936, lib.OPD_DTYPE_BF16, 1.0)
+    n = lib.opd_kl_workspace_size(p)
+    # dominated by the bf16 dz buffer of T x round_up(V, 64) elements
+    assert n >= 16384 * 151936 * 2 and n < 16384 * 151936 * 2 * 1.2
+    assert lib.opd_kl_workspace_size(lib.make_problem(64, 64, 128, 1000, lib.OPD_DTYPE_F32, 1.0)) > 64 * 1000 * 4
+    for bad in (lib.make_problem(-1, 8, 8, 8), lib.make_problem(8, 0, 8, 8), lib.make_problem(8, 8, 8, 0),
+                lib.make_problem(8, 8, 8, 8, 7), lib.make_problem(8, 8, 8, 8, 0, 0.0),
+                lib.make_problem(8, 8, 8, 8, 0, float("nan")), lib.make_problem(8, 12, 8, 8, 0)):
+        assert lib.opd_kl_workspace_size(bad) == 0
+
+
+def test_invalid_arguments_rejected_before_any_launch(lib):
+    vp = ctypes.c_void_p
+    fake = vp(1 << 20)  # never dereferenced: validation fails first
+    bad = lib.make_problem(8, 8, 8, 8, lib.OPD_DTYPE_BF16, -1.0)
+    rc = lib.call_raw("opd_kl_forward", ctypes.byref(bad), fake, fake, fake, fake, fake, fake, fake, fake,
+                      ctypes.c_size_t(1 << 20), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+    odd = lib.make_problem(8, 12, 8, 8, lib.OPD_DTYPE_BF16, 1.0)
+    rc = lib.call_raw("opd_kl_forward", ctypes.byref(odd), fake, fake, fake, fake, fake, fake, fake, fake,
+                      ctypes.c_size_t(1 << 20), None)
+    assert rc == lib.OPD_ERR_UNSUPPORTED
+    ok = lib.make_problem(8, 8, 8, 8, lib.OPD_DTYPE_BF16, 1.0)
+    rc = lib.call_raw("opd_kl_forward", ctypes.byref(ok), fake, fake, fake, fake, fake, fake, fake, None,
+                      ctypes.c_size_t(0), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG  # no workspace
+    rc = lib.call_raw("opd_kl_forward", ctypes.byref(ok), fake, fake, fake, fake, fake, fake, fake, vp(4096 + 8),
+                      ctypes.c_size_t(1 << 20), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG  # misaligned workspace
+    rc = lib.call_raw("opd_kl_forward", None, fake, fake, fake, fake, fake, fake, fake, fake,
+                      ctypes.c_size_t(1 << 20), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+    rc = lib.call_raw("opd_kl_selftest_timeout", fake, ctypes.c_size_t(1 << 20), ctypes.c_uint64(0), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+
+
+def test_seq_mean_token_mean_helper_matches_oracle(lib, oracle_mod):
+    from paper_2609_36608_gb300 import synth
+    for name in ("tiny_fp32", "qwen3_0p6b", "ragged_multiturn"):
+        lay = synth.layout(synth.WORKLOADS[name])
+        w = lib.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)
+        ref = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)
+        np.testing.assert_allclose(w, ref, rtol=2e-7, atol=0)
+    with pytest.raises(lib.OpdError):
+        lib.opd_seq_mean_token_mean_weights(np.zeros(3, np.int32), np.zeros(3, np.uint8), -1.0)

@@ -1,0 +1,219 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 CPU oracle.
+
+Tolerances (per-token KL and gradients of the reverse KL, Section 3
+Eq. reverse-kl): |KL_gpu - KL_oracle| <= 1e-4 + 2e-3 |KL_oracle| elementwise;
+dH_s and dW_s within 1e-2 relative Frobenius error (bf16 inputs, fp32
+accumulation, bf16 staging of dz). The float32 path is held to 1e-5 / 1e-4.
+
+Small cases run the whole oracle; full-size workloads run the bench's launch
+configuration and check a deterministic sample of rows (rows are independent
+given the hidden states), plus dW_s on a mask-subsetted full-shape run.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36608_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+KL_ABS, KL_REL, GRAD_REL = 1e-4, 2e-3, 1e-2
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+    return opd_kl
+
+
+def _rel(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _check_kl(got, want, abs_tol=KL_ABS, rel_tol=KL_REL):
+    excess = np.abs(np.asarray(got, np.float64) - want) - (abs_tol + rel_tol * np.abs(want))
+    assert excess.max() <= 0, f"KL worst excess {excess.max():.3e} at {int(excess.argmax())}"
+
+
+def _run(lib, w, x, mask, g, *, mode="fwd_bwd", accumulate=False, dW_init=None):
+    dev = x["H_s"].device
+    dtype = lib.OPD_DTYPE_F32 if w.dtype == "f32" else lib.OPD_DTYPE_BF16
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
+    ws = lib.allocate_workspace(prob, dev)
+    m = torch.as_tensor(mask, device=dev, dtype=torch.uint8)
+    grad = torch.as_tensor(np.asarray(g, np.float32), device=dev)
+    kl = torch.full((w.T,), float("nan"), device=dev)
+    stats = torch.full((w.T, 3), float("nan"), device=dev)
+    dH = torch.full((w.T, w.d_s), float("nan"), device=dev)
+    dW = torch.full((w.V, w.d_s), float("nan"), device=dev) if dW_init is None else dW_init.clone()
+    if mode == "fwd_bwd":
+        lib.opd_kl_fwd_bwd(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], m, grad, kl, stats, dH, dW, accumulate, ws)
+    else:
+        lib.opd_kl_forward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], m, kl, stats, ws)
+        lib.opd_kl_backward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], m, stats, grad, dH, dW, accumulate, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    return {"kl": kl.cpu().numpy(), "stats": stats.cpu().numpy(), "dH": dH.cpu().numpy(), "dW": dW.cpu().numpy()}
+
+
+def _host(x):
+    return [synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")]
+
+
+def _g64(g, mask):
+    # the GPU receives float32 weights; the oracle gets the same values widened
+    return np.where(np.asarray(mask) != 0, np.asarray(g, np.float32).astype(np.float64), 0.0)
+
+
+def _full_check(lib, oracle_mod, w, mask=None, g=None, tight=False, **kw):
+    lay = synth.layout(w) if mask is None else None
+    mask = lay.mask if mask is None else mask
+    g = synth.uniform_weights(w.seed, w.T) if g is None else g
+    x = synth.hidden_and_heads(w, "cuda")
+    out = _run(lib, w, x, mask, g, **kw)
+    ref = oracle_mod.opd_kl(*_host(x), mask, _g64(g, mask), w.tau)
+    if tight:
+        _check_kl(out["kl"], ref.kl, 1e-5, 1e-5)
+    else:
+        _check_kl(out["kl"], ref.kl)
+    sup = np.asarray(mask) != 0
+    assert (out["kl"][~sup] == 0).all() and (out["dH"][~sup] == 0).all()
+    np.testing.assert_allclose(out["stats"][sup, 0], ref.lse_s[sup], rtol=1e-5, atol=1e-4)
+    np.testing.assert_allclose(out["stats"][sup, 1], ref.lse_t[sup], rtol=1e-5, atol=1e-4)
+    lim = 1e-4 if tight else GRAD_REL
+    assert _rel(out["dH"], ref.dH_s) <= lim, _rel(out["dH"], ref.dH_s)
+    assert _rel(out["dW"], ref.dW_s) <= lim, _rel(out["dW"], ref.dW_s)
+    return out, ref, x
+
+
+@pytest.mark.parametrize("layout", ["tiny", "tiny_alt"])
+def test_tiny_fp32_config(lib, oracle_mod, layout):
+    w = synth.scaled(synth.WORKLOADS["tiny_fp32"], layout=layout)
+    _full_check(lib, oracle_mod, w, tight=True)
+
+
+def _small_bf16(**kw):
+    base = dict(name="small", T=700, d_s=256, d_t=384, V=1000, tau=0.7, n_traj=7, traj_len=100, seed=11)
+    base.update(kw)
+    return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
+
+
+def test_bf16_several_tiles_ragged_vocab(lib, oracle_mod):
+    # 3+ row tiles with a ragged last tile, 8 vocabulary tiles with a 104-column tail,
+    # K blocks 4 (student) and 6 (teacher)
+    _full_check(lib, oracle_mod, _small_bf16())
+
+
+def test_bf16_ragged_hidden_sizes_and_vocab(lib, oracle_mod):
+    # d not a multiple of the 64-wide K block, d_s not a multiple of the 256-wide GEMM tile,
+    # V not a multiple of 8 (dz pitch padding)
+    _full_check(lib, oracle_mod, _small_bf16(T=300, d_s=200, d_t=136, V=1237, tau=1.3, n_traj=3, seed=12))
+
+
+def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
+    w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
+                    seed=13)
+    out, ref, _ = _full_check(lib, oracle_mod, w)
+    sup = synth.layout(w).mask != 0
+    assert np.median(ref.kl[sup]) < 1.0
+
+
+def test_forward_then_backward_matches_fused_call(lib):
+    w = _small_bf16(T=400, seed=14)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    a = _run(lib, w, x, lay.mask, g, mode="fwd_bwd")
+    b = _run(lib, w, x, lay.mask, g, mode="separate")
+    np.testing.assert_array_equal(a["kl"], b["kl"])
+    np.testing.assert_array_equal(a["stats"], b["stats"])
+    assert _rel(b["dH"], a["dH"].astype(np.float64)) < 1e-5
+    assert _rel(b["dW"], a["dW"].astype(np.float64)) < 1e-5
+
+
+def test_accumulate_dW_adds(lib):
+    w = _small_bf16(T=300, seed=15)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    plain = _run(lib, w, x, lay.mask, g)
+    init = torch.randn(w.V, w.d_s, device="cuda", generator=torch.Generator("cuda").manual_seed(0))
+    acc = _run(lib, w, x, lay.mask, g, accumulate=True, dW_init=init)
+    assert _rel(acc["dW"] - init.cpu().numpy(), plain["dW"].astype(np.float64)) < 1e-5
+
+
+def test_all_rows_masked(lib):
+    w = _small_bf16(T=200, seed=16)
+    mask = np.zeros(w.T, np.uint8)
+    x = synth.hidden_and_heads(w, "cuda")
+    out = _run(lib, w, x, mask, np.ones(w.T))
+    assert (out["kl"] == 0).all() and (out["dH"] == 0).all() and (out["dW"] == 0).all()
+    init = torch.ones(w.V, w.d_s, device="cuda")
+    acc = _run(lib, w, x, mask, np.ones(w.T), accumulate=True, dW_init=init)
+    assert (acc["dW"] == 1).all()
+
+
+@pytest.mark.parametrize("rows", [[0], [199], [5, 6, 7, 127, 128, 129]])
+def test_few_supervised_rows(lib, oracle_mod, rows):
+    w = _small_bf16(T=200, seed=17)
+    mask = np.zeros(w.T, np.uint8)
+    mask[rows] = 1
+    _full_check(lib, oracle_mod, w, mask=mask)
+
+
+def test_student_equals_teacher_gives_zero(lib):
+    w = _small_bf16(T=256, d_t=256, seed=18)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    x["H_t"], x["W_t"] = x["H_s"], x["W_s"]
+    out = _run(lib, w, x, lay.mask, synth.uniform_weights(w.seed, w.T))
+    assert np.abs(out["kl"]).max() < 2e-5
+    # dz = p_s (log p_s - log p_t - KL) vanishes up to fp32 rounding of identical logits
+    assert np.abs(out["dH"]).max() < 1e-4 and np.abs(out["dW"]).max() < 1e-4
+
+
+def test_bounded_wait_timeout_reports_and_context_survives(lib):
+    prob = lib.make_problem(64, 64, 64, 64, lib.OPD_DTYPE_BF16, 1.0)
+    ws = lib.allocate_workspace(prob)
+    assert lib.opd_kl_selftest_timeout(ws, 50_000_000) == lib.OPD_ERR_TIMEOUT
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK  # status was cleared
+    w = _small_bf16(T=128, d_s=64, d_t=64, V=64, n_traj=1, traj_len=128, seed=19)
+    x = synth.hidden_and_heads(w, "cuda")
+    out = _run(lib, w, x, synth.layout(w).mask, np.ones(w.T))
+    assert np.isfinite(out["kl"]).all()
+
+
+FULL = ["qwen3_0p6b", "qwen3_1p7b", "qwen3_4b", "ragged_multiturn"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled_rows(lib, oracle_mod, name):
+    w = synth.WORKLOADS[name]
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    out = _run(lib, w, x, lay.mask, g)
+    sup = lay.mask != 0
+    # properties at any size
+    assert (out["kl"][~sup] == 0).all() and (out["dH"][~sup] == 0).all()
+    assert out["kl"][sup].min() > -1e-4 and np.isfinite(out["dW"]).all()
+    # sampled rows against the oracle
+    rows = np.flatnonzero(sup)
+    pick = np.unique(np.concatenate([rows[np.linspace(0, len(rows) - 1, 16).astype(int)], rows[:2], rows[-2:]]))
+    H_s, H_t, W_s, W_t = _host(x)
+    ref = oracle_mod.opd_kl(H_s, H_t, W_s, W_t, lay.mask, _g64(g, lay.mask), w.tau, rows=pick, want_dW=False)
+    _check_kl(out["kl"][pick], ref.kl)
+    assert _rel(out["dH"][pick], ref.dH_s) <= GRAD_REL
+    # dW_s on the same shapes with only a few supervised rows
+    sub = pick[::2]
+    mask2 = np.zeros_like(lay.mask)
+    mask2[sub] = 1
+    out2 = _run(lib, w, x, mask2, g)
+    ref2 = oracle_mod.opd_kl(H_s, H_t, W_s, W_t, mask2, _g64(g, mask2), w.tau, rows=sub, want_dH=False)
+    assert _rel(out2["dW"], ref2.dW_s) <= GRAD_REL, _rel(out2["dW"], ref2.dW_s)
+    _check_kl(out2["kl"][sub], ref2.kl)
