@@ -103,6 +103,30 @@ opd_status opd_kl_fwd_bwd(const opd_problem* problem, const void* H_s, const voi
                           float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
                           void* stream);
 
+/* Largest T that opd_kl_forward_noalloc accepts. */
+#define OPD_KL_NOALLOC_MAX_ROWS 4096
+
+/* opd_kl_forward without a workspace, for callers that cannot allocate device
+ * memory: hosts that own every byte of the GPU (a serving process or plugin host
+ * with a fixed pool) and do not let a library call cudaMalloc. The paper has no
+ * counterpart; this is a deployment convenience. Same inputs and outputs as
+ * opd_kl_forward (bf16 only), same results within the parity tolerance.
+ *   - Scratch is a fixed 5,259,520-byte array in the library's device memory,
+ *     held by every GPU that loads the library until the process exits.
+ *   - T above OPD_KL_NOALLOC_MAX_ROWS returns OPD_ERR_UNSUPPORTED (use
+ *     opd_kl_forward); F32 problems also return OPD_ERR_UNSUPPORTED.
+ *   - The first call on each device looks up the array's device address with
+ *     that device current; make that first call before any stream capture.
+ *   - All calls share the array, which keeps the last call's contents (each call
+ *     resets what must start at zero), so calls whose kernels overlap on the
+ *     GPU race on it: serialise them on one stream.
+ *   - Rows are not compacted: unsupervised rows are computed and then written
+ *     as zeros, so the tensor-core work scales with T rather than with the
+ *     supervised count.
+ * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
+opd_status opd_kl_forward_noalloc(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                                  const void* W_t, const uint8_t* mask, float* kl_out, float* stats, void* stream);
+
 /* Host helper (Appendix B.4, Eq. opd-surrogate, seq-mean-token-mean): upstream
  * weights w_i = dL/dl_i for L = 1/|B| sum_b (sum_j m_bj l_bj) / (sum_j m_bj + eps).
  * seg_id [T]: response index of row i (>= 0) or negative outside any response;

@@ -27,6 +27,8 @@ OPD_ERR_NONFINITE = 5
 OPD_DTYPE_BF16 = 0
 OPD_DTYPE_F32 = 1
 
+OPD_KL_NOALLOC_MAX_ROWS = 4096
+
 
 class opd_problem(ctypes.Structure):
     _fields_ = [("T", ctypes.c_int64), ("d_s", ctypes.c_int64), ("d_t", ctypes.c_int64), ("V", ctypes.c_int64),
@@ -53,6 +55,7 @@ def _load() -> ctypes.CDLL:
     sig = {
         "opd_kl_workspace_size": (sz, [P]),
         "opd_kl_forward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
+        "opd_kl_forward_noalloc": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp]),
         "opd_kl_backward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, sz, vp]),
         "opd_kl_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, sz, vp]),
         "opd_seq_mean_token_mean_weights": (i32, [vp, vp, i64, ctypes.c_float, vp]),
@@ -122,6 +125,14 @@ def opd_kl_forward(problem, H_s, H_t, W_s, W_t, mask, kl_out, stats, workspace, 
     _check(_lib.opd_kl_forward(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
                                _ptr(kl_out), _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream)),
            "opd_kl_forward")
+
+
+def opd_kl_forward_noalloc(problem, H_s, H_t, W_s, W_t, mask, kl_out, stats, stream=None) -> None:
+    """opd_kl_forward without a workspace, for callers that may not allocate device memory
+    (T <= OPD_KL_NOALLOC_MAX_ROWS, bf16; scratch is a fixed array inside the library)."""
+    _check(_lib.opd_kl_forward_noalloc(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t),
+                                       _ptr(mask), _ptr(kl_out), _ptr(stats), _stream(stream)),
+           "opd_kl_forward_noalloc")
 
 
 def opd_kl_backward(problem, H_s, H_t, W_s, W_t, mask, stats, grad_kl, dH_s, dW_s, accumulate_dW: bool,

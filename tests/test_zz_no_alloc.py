@@ -1,0 +1,78 @@
+"""The workspace-free forward entry point against the regular forward.
+
+opd_kl_forward_noalloc serves callers that may not allocate device memory at
+all, such as a host process that owns the whole GPU through its own fixed pool
+and forbids libraries from calling cudaMalloc. It keeps its scratch in a fixed
+array inside the library instead of a caller-provided workspace. This file
+checks it through the C ABI against opd_kl_forward, with the same tolerance as
+the parity tests, on two calls in a row with different problems (the second
+call reuses the array the first one left behind). It runs last so that a
+failure here leaves every other test already run.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36608_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+KL_ABS, KL_REL = 1e-4, 2e-3
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+    return opd_kl
+
+
+def _case(name, **kw):
+    base = dict(name=name, d_s=256, d_t=384, V=1000, tau=0.7, traj_len=100, n_traj=1)
+    base.update(kw)
+    return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
+
+
+def _both(lib, w):
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    mask = torch.from_numpy(lay.mask).cuda()
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    kl_ref = torch.full((w.T,), float("nan"), device="cuda")
+    st_ref = torch.full((w.T, 3), float("nan"), device="cuda")
+    lib.opd_kl_forward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, kl_ref, st_ref, ws)
+    kl = torch.full((w.T,), float("nan"), device="cuda")
+    st = torch.full((w.T, 3), float("nan"), device="cuda")
+    lib.opd_kl_forward_noalloc(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, kl, st)
+    torch.cuda.synchronize()
+    return lay.mask != 0, kl.cpu().numpy(), st.cpu().numpy(), kl_ref.cpu().numpy(), st_ref.cpu().numpy()
+
+
+def test_noalloc_forward_matches_workspace_forward_on_two_calls(lib):
+    cases = [_case("noalloc_a", T=700, seed=21),
+             _case("noalloc_b", T=lib.OPD_KL_NOALLOC_MAX_ROWS, d_s=128, d_t=192, V=1237, tau=1.0, seed=22,
+                   traj_len=512)]
+    for w in cases:
+        sup, kl, st, kl_ref, st_ref = _both(lib, w)
+        excess = np.abs(kl - kl_ref) - (KL_ABS + KL_REL * np.abs(kl_ref))
+        assert excess.max() <= 0, (w.name, float(excess.max()))
+        assert (kl[~sup] == 0).all() and (st[~sup] == 0).all()
+        np.testing.assert_allclose(st[sup], st_ref[sup], rtol=1e-5, atol=1e-4)
+
+
+def test_noalloc_rejects_rows_beyond_its_fixed_scratch(lib):
+    T = lib.OPD_KL_NOALLOC_MAX_ROWS + 1
+    prob = lib.make_problem(T, 64, 64, 128, lib.OPD_DTYPE_BF16, 1.0)
+    H = torch.zeros(T, 64, dtype=torch.bfloat16, device="cuda")
+    W = torch.zeros(128, 64, dtype=torch.bfloat16, device="cuda")
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    out = torch.empty(T, device="cuda")
+    stats = torch.empty(T, 3, device="cuda")
+    with pytest.raises(lib.OpdError) as e:
+        lib.opd_kl_forward_noalloc(prob, H, H, W, W, mask, out, stats)
+    assert e.value.status == lib.OPD_ERR_UNSUPPORTED
