@@ -260,15 +260,22 @@ struct Maps {
   CUtensorMap dz_a_mn, hsg_b_mn, dw; // dW_s GEMM
 };
 
+// Fused tile width: OPD_KL_FUSED_BN=128 or 256 overrides the default.
+int fused_tile_bn() {
+  const int v = env_int("OPD_KL_FUSED_BN", 0);
+  return (v == 128 || v == 256) ? v : kFusedBN;
+}
+
 opd_status encode_maps(const Call& c, const void* W_s, const void* W_t, float* dW_s, Maps& m, bool bwd) {
+  const uint32_t bn = (uint32_t)fused_tile_bn();
   const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
   const uint64_t Tp = (uint64_t)c.L.T_pad, ds = (uint64_t)c.p.d_s, dt = (uint64_t)c.p.d_t, V = (uint64_t)c.p.V;
   const uint64_t Vp = (uint64_t)c.L.Vp;
   bool ok = tmap2d(&m.hs, BF, 2, c.ws + c.L.hs_g, ds, Tp, ds, kKBlock, kRowTile) &&
             tmap2d(&m.ht, BF, 2, c.ws + c.L.ht_g, dt, Tp, dt, kKBlock, kRowTile) &&
-            tmap2d(&m.ws, BF, 2, W_s, ds, V, ds, kKBlock, kFusedBN) &&
-            tmap2d(&m.wt, BF, 2, W_t, dt, V, dt, kKBlock, kFusedBN);
+            tmap2d(&m.ws, BF, 2, W_s, ds, V, ds, kKBlock, bn) &&
+            tmap2d(&m.wt, BF, 2, W_t, dt, V, dt, kKBlock, bn);
   if (ok && bwd) {
     ok = tmap2d(&m.dz_store, BF, 2, c.ws + c.L.dz, V, Tp, Vp, 64, 32) &&
          tmap2d(&m.dz_a_k, BF, 2, c.ws + c.L.dz, V, Tp, Vp, kKBlock, kRowTile) &&
@@ -294,6 +301,7 @@ FusedParams fused_params(const Call& c) {
   fp.wait_limit_ns = kDefaultWaitLimitNs;
   fp.partials = reinterpret_cast<float*>(c.ws + c.L.partials);
   fp.rowc = reinterpret_cast<const float4*>(c.ws + c.L.rowc);
+  fp.bn = fused_tile_bn();
   return fp;
 }
 

@@ -22,16 +22,24 @@ namespace opd {
 
 namespace {
 
-template <int BN, bool BWD>
+// BN vocabulary columns per tile; NEPI epilogue warps (4, or 8 with two warps
+// per TMEM lane quadrant, each taking half of the tile's columns).
+template <int BN, bool BWD, int NEPI>
 struct FusedCfg {
   static constexpr int kBufs = 512 / (2 * BN);  // (student, teacher) accumulator pairs in TMEM
+  static constexpr int kHalves = NEPI / 4;      // epilogue warps per lane quadrant
+  static constexpr int kColsPerWarp = BN / kHalves;
+  static constexpr int kThreads = 64 + 32 * NEPI;
   static constexpr int kStages = BWD ? (BN == 128 ? 5 : 3) : (BN == 128 ? 6 : 4);
   static constexpr uint32_t kABytes = kRowTile * kKBlock * 2;
   static constexpr uint32_t kBBytes = BN * kKBlock * 2;
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
-  static constexpr uint32_t kStagingPerWarp = BWD ? 32 * BN * 2 : 0;  // bf16 dz rows of one warp
+  static constexpr uint32_t kStagingPerWarp = BWD ? 32 * kColsPerWarp * 2 : 0;  // bf16 dz rows of one warp
+  static constexpr uint32_t kMergeBytes = (!BWD && kHalves > 1) ? 4 * 5 * 32 * 4 : 0;  // per quadrant 5 x 32
   static constexpr uint32_t kBarrierBytes = 256;
-  static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 4 * kStagingPerWarp + kBarrierBytes;
+  static constexpr size_t kSmem =
+      1024 + (size_t)kStages * kStageBytes + NEPI * kStagingPerWarp + kMergeBytes + kBarrierBytes;
+  static_assert(kColsPerWarp % 64 == 0, "whole 64-column boxes per epilogue warp");
 };
 
 // Unit u -> (row tile, vocabulary tile range). Units are grouped by `G` row tiles
@@ -91,6 +99,7 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, 
 
 // Fold 32 columns (or the first nvalid of them) of one row into the running
 // base-2 statistics; indices stay compile-time so the values stay in registers.
+// x = z k2 with k2 = log2(e) / tau; A is kept in raw logit units (times k2 at the end).
 template <bool PARTIAL>
 __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint32_t (&rt)[32], int nvalid, float k2,
                                            float& ms, float& Ss, float& A, float& mt, float& St) {
@@ -114,32 +123,35 @@ __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint3
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
     if (!PARTIAL || j < nvalid) {
-      const float xs = __uint_as_float(rs[j]) * k2;
-      const float xt = __uint_as_float(rt[j]) * k2;
-      const float e = exp2f(xs - ms);
+      const float zs = __uint_as_float(rs[j]);
+      const float zt = __uint_as_float(rt[j]);
+      const float e = exp2f(fmaf(zs, k2, -ms));
       Ss += e;
-      A = fmaf(e, xs - xt, A);
-      St += exp2f(xt - mt);
+      A = fmaf(e, zs - zt, A);
+      St += exp2f(fmaf(zt, k2, -mt));
     }
   }
 }
 
-template <int BN, bool BWD>
-__global__ void __launch_bounds__(192, 1)
+template <int BN, bool BWD, int NEPI>
+__global__ void __launch_bounds__(64 + 32 * NEPI, 1)
     k_fused_logits(const __grid_constant__ CUtensorMap tm_hs, const __grid_constant__ CUtensorMap tm_ht,
                    const __grid_constant__ CUtensorMap tm_ws, const __grid_constant__ CUtensorMap tm_wt,
                    const __grid_constant__ CUtensorMap tm_dz, const FusedParams p) {
-  using C = FusedCfg<BN, BWD>;
+  using C = FusedCfg<BN, BWD, NEPI>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* stage_base = smem;
   uint8_t* staging = smem + C::kStages * C::kStageBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(staging + 4 * C::kStagingPerWarp);
+  float* merge = reinterpret_cast<float*>(staging + NEPI * C::kStagingPerWarp);
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(merge) + C::kMergeBytes);
   uint64_t* empty = full + C::kStages;
   uint64_t* acc_full = empty + C::kStages;
   uint64_t* acc_empty = acc_full + C::kBufs;
   uint64_t* mma_done = acc_empty + C::kBufs;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint64_t* merge_full = mma_done + 1;   // [4], forward with two warps per quadrant
+  uint64_t* merge_empty = merge_full + 4;  // [4]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(merge_empty + 4);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -153,9 +165,13 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int b = 0; b < C::kBufs; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 4);
+      mbar_init(&acc_empty[b], NEPI);
     }
     mbar_init(mma_done, 1);
+    for (int qd = 0; qd < 4; ++qd) {
+      mbar_init(&merge_full[qd], 1);
+      mbar_init(&merge_empty[qd], 1);
+    }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -270,19 +286,28 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int ew = warp - 2;                 // epilogue warp index
+    const int q = warp & 3;                  // TMEM lane quadrant this warp may access
+    const int half = ew / 4;                 // which share of the tile's columns
+    const int cbase = half * C::kColsPerWarp;
     const int row_in_tile = q * 32 + lane;
     const uint32_t t_lane = (uint32_t)(q * 32) << 16;
-    int lt = 0;
+    int lt = 0, nu = 0;
     bool ok = true;
-    uint8_t* stg = staging + q * C::kStagingPerWarp;
-    for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x) {
+    uint8_t* stg = staging + ew * C::kStagingPerWarp;
+    for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x, ++nu) {
       int rt, split, vb, ve;
       sch.unit(u, rt, split, vb, ve);
       const int row = rt * kRowTile + row_in_tile;
       float ms = -INFINITY, Ss = 0.f, A = 0.f, mt = -INFINITY, St = 0.f;
-      float4 rc = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (BWD) rc = p.rowc[row];
+      // backward row constants: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc)
+      float b1 = 0.f, kc = 0.f, cc = 0.f;
+      if (BWD) {
+        const float4 rc = p.rowc[row];
+        b1 = rc.x;
+        kc = rc.z * p.inv_tau;
+        cc = rc.z * rc.y;
+      }
       for (int vt = vb; vt < ve; ++vt, ++lt) {
         const int buf = lt % C::kBufs;
         const uint32_t acc_par = (uint32_t)(lt / C::kBufs) & 1u;
@@ -292,11 +317,11 @@ __global__ void __launch_bounds__(192, 1)
           break;
         }
         tc_fence_after();
-        const int col0 = vt * BN;
-        const uint32_t ts = tmem_base + t_lane + (uint32_t)(buf * 2 * BN);
+        const int col0 = vt * BN + cbase;
+        const uint32_t ts = tmem_base + t_lane + (uint32_t)(buf * 2 * BN + cbase);
         const uint32_t tt = ts + BN;
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = 0; c < C::kColsPerWarp / 32; ++c) {
           uint32_t rs[32], rtt[32];
           tmem_ld32x2(ts + c * 32, tt + c * 32, rs, rtt);
           if (!BWD) {
@@ -306,9 +331,9 @@ __global__ void __launch_bounds__(192, 1)
             else if (nvalid > 0)
               fold_chunk<true>(rs, rtt, nvalid, p.k2, ms, Ss, A, mt, St);
           } else {
-            const int h = c >> 1;  // 64-column box of the staging tile
+            const int h = c >> 1;  // 64-column box of this warp's staging tile
             if ((c & 1) == 0) {
-              if (lane == 0) bulk_wait_read<BN / 64 - 1>();
+              if (lane == 0) bulk_wait_read<C::kColsPerWarp / 64 - 1>();
               __syncwarp();
             }
             uint32_t w[16];
@@ -319,9 +344,8 @@ __global__ void __launch_bounds__(192, 1)
               for (int e = 0; e < 2; ++e) {
                 const float zs = __uint_as_float(rs[2 * j + e]);
                 const float zt = __uint_as_float(rtt[2 * j + e]);
-                const float ps = exp2f(fmaf(zs, p.k2, -rc.x));
-                const float dd = fmaf(zs - zt, p.inv_tau, -rc.y);
-                dz2[e] = rc.z * ps * dd;
+                const float ps = exp2f(fmaf(zs, p.k2, -b1));
+                dz2[e] = ps * fmaf(zs - zt, kc, -cc);
               }
               w[j] = pack_bf16x2(dz2[0], dz2[1]);
             }
@@ -347,6 +371,41 @@ __global__ void __launch_bounds__(192, 1)
         if (lane == 0) mbar_arrive(&acc_empty[buf]);
       }
       if (!BWD && ok) {
+        A *= p.k2;  // A was accumulated in raw logit units
+        if (C::kHalves > 1) {
+          // the two warps of a quadrant fold their column shares: half 1 hands its
+          // statistics to half 0 through shared memory
+          float* mb = merge + q * 5 * 32;
+          if (half == 1) {
+            if (nu > 0 && !__all_sync(0xffffffffu, mbar_wait(&merge_empty[q], (uint32_t)(nu - 1) & 1u, status, lim))) {
+              ok = false;
+              break;
+            }
+            mb[0 * 32 + lane] = ms;
+            mb[1 * 32 + lane] = Ss;
+            mb[2 * 32 + lane] = A;
+            mb[3 * 32 + lane] = mt;
+            mb[4 * 32 + lane] = St;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&merge_full[q]);
+            continue;
+          }
+          if (!__all_sync(0xffffffffu, mbar_wait(&merge_full[q], (uint32_t)nu & 1u, status, lim))) {
+            ok = false;
+            break;
+          }
+          const float ms1 = mb[0 * 32 + lane], Ss1 = mb[1 * 32 + lane], A1 = mb[2 * 32 + lane];
+          const float mt1 = mb[3 * 32 + lane], St1 = mb[4 * 32 + lane];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&merge_empty[q]);
+          const float Ms = fmaxf(ms, ms1), Mt = fmaxf(mt, mt1);
+          const float f0 = exp2f(ms - Ms), f1 = exp2f(ms1 - Ms);
+          Ss = Ss * f0 + Ss1 * f1;
+          A = A * f0 + A1 * f1;
+          St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
+          ms = Ms;
+          mt = Mt;
+        }
         const size_t plane = (size_t)p.T_pad;
         float* base = p.partials + (size_t)split * 5 * plane + row;
         base[0 * plane] = ms;
@@ -367,30 +426,41 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
-template <int BN, bool BWD>
+template <int BN, bool BWD, int NEPI>
 cudaError_t launch_fused_impl(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                               const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
                               cudaStream_t s) {
-  using C = FusedCfg<BN, BWD>;
+  using C = FusedCfg<BN, BWD, NEPI>;
   static_assert(C::kSmem <= 232448, "shared memory budget");
-  auto kern = k_fused_logits<BN, BWD>;
+  auto kern = k_fused_logits<BN, BWD, NEPI>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, 192, C::kSmem, s>>>(hs, ht, ws, wt, dz, p);
+  kern<<<grid, C::kThreads, C::kSmem, s>>>(hs, ht, ws, wt, dz, p);
   return cudaGetLastError();
+}
+
+template <bool BWD>
+cudaError_t launch_fused_bn(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
+                            const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
+                            cudaStream_t s) {
+  switch (fused_bn(p)) {
+    case 128: return launch_fused_impl<128, BWD, 4>(hs, ht, ws, wt, dz, p, grid, s);
+    case 256: return launch_fused_impl<256, BWD, 8>(hs, ht, ws, wt, dz, p, grid, s);
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
 
 cudaError_t launch_fused_forward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                  const CUtensorMap& wt, const FusedParams& p, int grid, cudaStream_t s) {
-  return launch_fused_impl<kFusedBN, false>(hs, ht, ws, wt, hs, p, grid, s);
+  return launch_fused_bn<false>(hs, ht, ws, wt, hs, p, grid, s);
 }
 
 cudaError_t launch_fused_backward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                   const CUtensorMap& wt, const CUtensorMap& dz_store, const FusedParams& p,
                                   int grid, cudaStream_t s) {
-  return launch_fused_impl<kFusedBN, true>(hs, ht, ws, wt, dz_store, p, grid, s);
+  return launch_fused_bn<true>(hs, ht, ws, wt, dz_store, p, grid, s);
 }
 
 }  // namespace opd

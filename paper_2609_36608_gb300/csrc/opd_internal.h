@@ -15,7 +15,7 @@ constexpr int kRowTile = 128;   // token rows per MMA tile (TMEM lanes)
 constexpr int kKBlock = 64;     // bf16 elements per 128-byte swizzled row
 constexpr int kMaxVSplit = 64;  // vocabulary splits of the forward statistics
 constexpr int kMaxKSplit = 16;  // K splits of the dH_s GEMM
-constexpr int kFusedBN = 128;   // vocabulary columns per fused tile
+constexpr int kFusedBN = 256;   // default vocabulary columns per fused tile (128 or 256)
 constexpr int kGemmBN = 256;    // output columns per gradient-GEMM tile
 
 struct FusedParams {
@@ -28,7 +28,12 @@ struct FusedParams {
   uint64_t wait_limit_ns;
   float* partials;      // forward: [kMaxVSplit][5][T_pad]
   const float4* rowc;   // backward: [T_pad] = (lse_s log2 e, lse_s - lse_t + KL, g / tau, 0)
+  int32_t bn;           // vocabulary columns per tile: 128 or 256 (0 = kFusedBN); the W tensor
+                        // maps must use the same box height
 };
+
+// Tile width the fused kernels use for these parameters.
+inline int fused_bn(const FusedParams& p) { return p.bn == 0 ? kFusedBN : p.bn; }
 
 struct GemmParams {
   Ctrl* ctrl;

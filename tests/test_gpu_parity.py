@@ -103,16 +103,29 @@ def _small_bf16(**kw):
     return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
 
 
-def test_bf16_several_tiles_ragged_vocab(lib, oracle_mod):
-    # 3+ row tiles with a ragged last tile, 8 vocabulary tiles with a 104-column tail,
+@pytest.fixture(params=[128, 256], ids=["bn128", "bn256"])
+def fused_bn(request, monkeypatch):
+    """Both vocabulary tile widths of the fused kernels (the library reads the override per call)."""
+    monkeypatch.setenv("OPD_KL_FUSED_BN", str(request.param))
+    return request.param
+
+
+def test_bf16_several_tiles_ragged_vocab(lib, oracle_mod, fused_bn):
+    # 3+ row tiles with a ragged last tile, several vocabulary tiles with a ragged tail,
     # K blocks 4 (student) and 6 (teacher)
     _full_check(lib, oracle_mod, _small_bf16())
 
 
-def test_bf16_ragged_hidden_sizes_and_vocab(lib, oracle_mod):
+def test_bf16_ragged_hidden_sizes_and_vocab(lib, oracle_mod, fused_bn):
     # d not a multiple of the 64-wide K block, d_s not a multiple of the 256-wide GEMM tile,
     # V not a multiple of 8 (dz pitch padding)
     _full_check(lib, oracle_mod, _small_bf16(T=300, d_s=200, d_t=136, V=1237, tau=1.3, n_traj=3, seed=12))
+
+
+def test_bf16_many_vocab_splits(lib, oracle_mod, fused_bn):
+    # few row tiles and a long vocabulary: the forward splits V across many CTAs
+    _full_check(lib, oracle_mod, _small_bf16(T=256, d_s=64, d_t=64, V=40000, tau=1.0, n_traj=2, traj_len=128,
+                                             seed=23))
 
 
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
@@ -159,7 +172,7 @@ def test_all_rows_masked(lib):
 
 
 @pytest.mark.parametrize("rows", [[0], [199], [5, 6, 7, 127, 128, 129]])
-def test_few_supervised_rows(lib, oracle_mod, rows):
+def test_few_supervised_rows(lib, oracle_mod, rows, fused_bn):
     w = _small_bf16(T=200, seed=17)
     mask = np.zeros(w.T, np.uint8)
     mask[rows] = 1
