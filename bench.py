@@ -68,7 +68,7 @@ def load_peaks():
 # --------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) of the benchmarked GPU while the timed region runs."""
+    """nvidia-smi samples (every 50 ms) of the benchmarked GPU while the timed region runs."""
 
     FIELDS = ["clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
               "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
@@ -88,7 +88,7 @@ class ClockSampler:
             vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
             ident = vis.split(",")[device_index] if vis else str(device_index)
         self.cmd = [exe, "-i", ident, "--query-gpu=" + ",".join(self.FIELDS), "--format=csv,noheader,nounits",
-                    "-lms", "200"]
+                    "-lms", "50"]
 
     def start(self):
         if not hasattr(self, "cmd"):
@@ -285,16 +285,16 @@ def run_gpu(args):
     def step(H_s, H_t, m, gr):
         opd_kl.opd_kl_fwd_bwd(prob, H_s, H_t, x["W_s"], x["W_t"], m, gr, kl, stats, dH, dW, False, ws)
 
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
     for _ in range(args.warmup):
         step(x["H_s"], x["H_t"], mask, grad)
     torch.cuda.synchronize()
     if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
         raise RuntimeError("device status after warm-up is not OK")
-
-    sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
-        sampler.start()
-        time.sleep(0.3)
+        sampler.rows.clear()  # keep only samples taken while the timed steps run
     barrier(world)
     torch.cuda.synchronize()
     opd_kl.opd_kl_profile_start()
@@ -409,6 +409,58 @@ def run_gpu(args):
     return 0
 
 
+def run_calibration(args):
+    """Sustained comparison under the board power cap: cuBLAS bf16 8192^3 (torch.matmul, a library
+    reference point, not part of the step), then the fused step and the forward alone, each for
+    args.calibrate seconds with clocks and power sampled every 50 ms. One JSON line per run."""
+    if not torch.cuda.is_available():
+        raise SystemExit("--calibrate needs a CUDA GPU")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+
+    def sustained(name, fn, flops):
+        fn()
+        torch.cuda.synchronize()
+        sampler = ClockSampler(0)
+        sampler.start()
+        n, t0 = 0, time.time()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        while time.time() - t0 < args.calibrate:
+            for _ in range(4):
+                fn()
+            n += 4
+            torch.cuda.synchronize()
+        e1.record()
+        torch.cuda.synchronize()
+        sampler.stop()
+        ms = e0.elapsed_time(e1)
+        print(json.dumps({"calibration": name, "calls": n, "ms_per_call": ms / n,
+                          "tflops": flops * n / (ms / 1e3) / 1e12, "clocks": sampler.summary()}), flush=True)
+
+    a = torch.randn(8192, 8192, device="cuda", dtype=torch.bfloat16)
+    b = torch.randn(8192, 8192, device="cuda", dtype=torch.bfloat16)
+    sustained("cublas_bf16_8192", lambda: torch.matmul(a, b), 2.0 * 8192 ** 3)
+    del a, b
+    w = synth.WORKLOADS[args.workload]
+    lay = synth.layout(w)
+    R = int(lay.mask.sum())
+    x = synth.hidden_and_heads(w, "cuda")
+    prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, opd_kl.OPD_DTYPE_BF16, w.tau)
+    ws = opd_kl.allocate_workspace(prob)
+    mask = torch.from_numpy(lay.mask).cuda()
+    grad = torch.from_numpy(opd_kl.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask)).cuda()
+    kl, st = torch.empty(w.T, device="cuda"), torch.empty(w.T, 3, device="cuda")
+    dH, dW = torch.empty(w.T, w.d_s, device="cuda"), torch.empty(w.V, w.d_s, device="cuda")
+    executed, _ = step_flops(w, R)
+    sustained(f"fwd_bwd_{w.name}", lambda: opd_kl.opd_kl_fwd_bwd(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"],
+                                                                 mask, grad, kl, st, dH, dW, False, ws), executed)
+    sustained(f"fwd_{w.name}", lambda: opd_kl.opd_kl_forward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask,
+                                                             kl, st, ws), 2.0 * R * w.V * (w.d_s + w.d_t))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -419,7 +471,11 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
     ap.add_argument("--ref-rows", type=int, default=8, help="rows per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--calibrate", type=float, default=0.0, metavar="SECONDS",
+                    help="instead of the benchmark: sustained cuBLAS vs fused-step runs under the power cap")
     args = ap.parse_args()
+    if args.calibrate > 0:
+        return run_calibration(args)
     if args.warmup < 3:
         log("note: at least 3 warm-up steps are required for a valid measurement; using 3")
         args.warmup = 3

@@ -31,7 +31,7 @@ struct WsLayout {
 // Workspace layout, 256-byte aligned sections. Sized for every row supervised.
 WsLayout ws_layout(const opd_problem& p) {
   WsLayout L;
-  L.T_pad = (int64_t)round_up((size_t)(p.T > 0 ? p.T : 1), kRowTile);
+  L.T_pad = (int64_t)round_up((size_t)(p.T > 0 ? p.T : 1), kRowPad);
   L.Vp = (int64_t)round_up((size_t)p.V, 64);
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -260,14 +260,16 @@ struct Maps {
   CUtensorMap dz_a_mn, hsg_b_mn, dw; // dW_s GEMM
 };
 
-// Fused tile width: OPD_KL_FUSED_BN=128 or 256 overrides the default.
-int fused_tile_bn() {
-  const int v = env_int("OPD_KL_FUSED_BN", 0);
-  return (v == 128 || v == 256) ? v : kFusedBN;
+// Fused-kernel tiling: OPD_KL_FUSED=bn256 | pair256 overrides the default.
+int fused_tile_mode() {
+  const char* v = std::getenv("OPD_KL_FUSED");
+  if (v && std::strcmp(v, "bn256") == 0) return kFusedBN256;
+  if (v && std::strcmp(v, "pair256") == 0) return kFusedPair256;
+  return kFusedDefaultMode;
 }
 
 opd_status encode_maps(const Call& c, const void* W_s, const void* W_t, float* dW_s, Maps& m, bool bwd) {
-  const uint32_t bn = (uint32_t)fused_tile_bn();
+  const uint32_t bn = (uint32_t)fused_w_box(fused_tile_mode());
   const auto BF = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
   const auto F32 = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
   const uint64_t Tp = (uint64_t)c.L.T_pad, ds = (uint64_t)c.p.d_s, dt = (uint64_t)c.p.d_t, V = (uint64_t)c.p.V;
@@ -301,7 +303,8 @@ FusedParams fused_params(const Call& c) {
   fp.wait_limit_ns = kDefaultWaitLimitNs;
   fp.partials = reinterpret_cast<float*>(c.ws + c.L.partials);
   fp.rowc = reinterpret_cast<const float4*>(c.ws + c.L.rowc);
-  fp.bn = fused_tile_bn();
+  fp.mode = fused_tile_mode();
+  fp.max_vsplit = kMaxVSplit;
   return fp;
 }
 

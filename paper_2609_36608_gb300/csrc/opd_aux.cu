@@ -70,7 +70,7 @@ __global__ void k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict_
                           const int32_t* __restrict__ idx, const Ctrl* __restrict__ ctrl, uint4* __restrict__ Hs_g,
                           uint4* __restrict__ Ht_g) {
   const int R = ctrl->R;
-  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  const int R_pad = (R + kRowPad - 1) / kRowPad * kRowPad;
   const int per_row = vs + vt;
   const long total = (long)R_pad * per_row;
   for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x) {
@@ -130,7 +130,7 @@ __global__ void k_bwd_rowc(const float* __restrict__ stats, const float* __restr
                            const int32_t* __restrict__ idx, const Ctrl* __restrict__ ctrl, int32_t T_pad, float tau,
                            float4* __restrict__ rowc) {
   const int R = ctrl->R;
-  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  const int R_pad = (R + kRowPad - 1) / kRowPad * kRowPad;
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R_pad; r += gridDim.x * blockDim.x) {
     float4 c = make_float4(0.f, 0.f, 0.f, 0.f);
     if (r < R) {
@@ -148,7 +148,7 @@ __global__ void k_bwd_rowc(const float* __restrict__ stats, const float* __restr
 
 __global__ void k_zero_rows(float4* __restrict__ buf, int32_t vec_per_row, const Ctrl* __restrict__ ctrl) {
   const int R = ctrl->R;
-  const int R_pad = (R + kRowTile - 1) / kRowTile * kRowTile;
+  const int R_pad = (R + kRowPad - 1) / kRowPad * kRowPad;
   const long total = (long)R_pad * vec_per_row;
   for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x)
     buf[e] = make_float4(0.f, 0.f, 0.f, 0.f);

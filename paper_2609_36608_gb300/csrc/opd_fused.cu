@@ -1,8 +1,8 @@
 // Fused vocabulary-tiled LM-head kernel (tcgen05 + TMEM + TMA), two variants:
 //
-//  forward  (Section 3, Eq. reverse-kl): for a tile of 128 supervised token rows
-//           and BN vocabulary columns, the student logits z_s = H_s W_s^T and the
-//           teacher logits z_t = H_t W_t^T accumulate in TMEM; the epilogue folds
+//  forward  (Section 3, Eq. reverse-kl): for a tile of supervised token rows and
+//           256 vocabulary columns, the teacher logits z_t = H_t W_t^T and the
+//           student logits z_s = H_s W_s^T accumulate in TMEM; the epilogue folds
 //           them into per-row online statistics in base 2 (x = z log2(e) / tau):
 //             m_s, S_s = sum 2^(x_s - m_s), A = sum 2^(x_s - m_s) (x_s - x_t),
 //             m_t, S_t = sum 2^(x_t - m_t)
@@ -12,9 +12,23 @@
 //           (the derivative of g KL with respect to the student logits) as bf16
 //           for the two gradient GEMMs.
 //
-// Roles (192 threads): warp 0 issues TMA loads, warp 1 allocates TMEM and issues
-// the MMAs from one thread, warps 2-5 run the epilogue (one TMEM lane = one row).
-// Persistent: each CTA walks work units (row tile, vocabulary range) grid-strided.
+// Roles: warp 0 issues TMA loads, warp 1 allocates TMEM and issues the MMAs from
+// one thread, eight epilogue warps drain TMEM (TMEM lane = tile row; the two
+// warps of each lane quadrant take 128 columns each). Persistent: work units (row
+// tile, vocabulary range) are walked grid-strided.
+//
+// TMEM holds one tile: teacher accumulator in columns [0,256), student in
+// [256,512). Each tile computes the teacher segment first. The epilogue copies
+// its teacher columns to registers and releases them at once, so the next tile's
+// teacher GEMM (d_t of the d_s + d_t reduction) overlaps this tile's epilogue;
+// the student columns are released as soon as they have been read, well before
+// the next tile's student GEMM starts.
+//
+// PAIR = true runs each tile on a CTA pair (2-CTA cluster, tcgen05 cta_group::2):
+// 256 rows per tile, 128 in each CTA's TMEM; each CTA stages its own 128 rows of
+// H and 128 of the 256 rows of W, the even-ranked CTA issues the MMAs, and both
+// CTAs' TMA completions are counted on the leader's barriers. Per byte staged
+// from L2 this does twice the MMA work of a single-CTA 128 x 256 tile.
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
@@ -22,45 +36,49 @@ namespace opd {
 
 namespace {
 
-// BN vocabulary columns per tile; NEPI epilogue warps (4, or 8 with two warps
-// per TMEM lane quadrant, each taking half of the tile's columns).
-template <int BN, bool BWD, int NEPI>
+constexpr int kBN = 256;   // vocabulary columns per tile (MMA N)
+constexpr int kNEpi = 8;   // epilogue warps
+constexpr int kColsPerWarp = kBN / 2;
+constexpr int kThreads = 64 + 32 * kNEpi;
+
+template <bool BWD, bool PAIR>
 struct FusedCfg {
-  static constexpr int kBufs = 512 / (2 * BN);  // (student, teacher) accumulator pairs in TMEM
-  static constexpr int kHalves = NEPI / 4;      // epilogue warps per lane quadrant
-  static constexpr int kColsPerWarp = BN / kHalves;
-  static constexpr int kThreads = 64 + 32 * NEPI;
-  static constexpr int kStages = BWD ? (BN == 128 ? 5 : 3) : (BN == 128 ? 6 : 4);
+  static constexpr int kTileRows = PAIR ? 2 * kRowTile : kRowTile;  // rows per tile (whole pair)
+  static constexpr int kBRows = PAIR ? kBN / 2 : kBN;              // W rows staged by one CTA
   static constexpr uint32_t kABytes = kRowTile * kKBlock * 2;
-  static constexpr uint32_t kBBytes = BN * kKBlock * 2;
+  static constexpr uint32_t kBBytes = kBRows * kKBlock * 2;
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
   static constexpr uint32_t kStagingPerWarp = BWD ? 32 * kColsPerWarp * 2 : 0;  // bf16 dz rows of one warp
-  static constexpr uint32_t kMergeBytes = (!BWD && kHalves > 1) ? 4 * 5 * 32 * 4 : 0;  // per quadrant 5 x 32
+  static constexpr uint32_t kMergeBytes = BWD ? 0 : 4 * 5 * 32 * 4;             // per quadrant 5 x 32
   static constexpr uint32_t kBarrierBytes = 256;
-  static constexpr size_t kSmem =
-      1024 + (size_t)kStages * kStageBytes + NEPI * kStagingPerWarp + kMergeBytes + kBarrierBytes;
-  static_assert(kColsPerWarp % 64 == 0, "whole 64-column boxes per epilogue warp");
+  static constexpr size_t kFixed = 1024 + (size_t)kNEpi * kStagingPerWarp + kMergeBytes + kBarrierBytes;
+  static constexpr int kStagesFit = (int)((232448 - kFixed) / kStageBytes);
+  static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
+  static constexpr size_t kSmem = kFixed + (size_t)kStages * kStageBytes;
+  static constexpr int kFreeCount = PAIR ? 2 * kNEpi : kNEpi;  // epilogue warps that release TMEM
+  static_assert(kStages >= 3, "pipeline depth");
 };
 
 // Unit u -> (row tile, vocabulary tile range). Units are grouped by `G` row tiles
-// so that CTAs running at the same time share a few hidden-state tiles and a few
-// vocabulary tiles in L2.
+// so that CTAs (or CTA pairs) running at the same time share a few hidden-state
+// tiles and a few vocabulary tiles in L2.
 struct FusedSchedule {
   int n_rt, n_vt, n_vs, G, n_units;
 
-  __device__ void init(int R, int V, int BN, int grid, int G_, bool bwd) {
-    n_rt = (R + kRowTile - 1) / kRowTile;
-    n_vt = (V + BN - 1) / BN;
+  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split, bool bwd) {
+    n_rt = (R + tile_rows - 1) / tile_rows;
+    n_vt = (V + kBN - 1) / kBN;
     G = G_ < 1 ? 1 : G_;
     if (bwd || n_rt == 0) {
       n_vs = bwd ? n_vt : 1;
     } else {
-      // fewest tiles on the busiest CTA, then the fewest splits
+      // fewest tiles on the busiest worker, then the fewest splits
       long best = -1;
       n_vs = 1;
-      const int max_vs = n_vt < kMaxVSplit ? n_vt : kMaxVSplit;
+      const int cap = max_split < 1 ? 1 : (max_split > kMaxVSplit ? kMaxVSplit : max_split);
+      const int max_vs = n_vt < cap ? n_vt : cap;
       for (int s = 1; s <= max_vs; ++s) {
-        const long waves = ((long)n_rt * s + grid - 1) / grid;
+        const long waves = ((long)n_rt * s + workers - 1) / workers;
         const long cost = waves * ((n_vt + s - 1) / s);
         if (best < 0 || cost < best) {
           best = cost;
@@ -98,17 +116,18 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, 
 }
 
 // Fold 32 columns (or the first nvalid of them) of one row into the running
-// base-2 statistics; indices stay compile-time so the values stay in registers.
-// x = z k2 with k2 = log2(e) / tau; A is kept in raw logit units (times k2 at the end).
-template <bool PARTIAL>
-__device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint32_t (&rt)[32], int nvalid, float k2,
-                                           float& ms, float& Ss, float& A, float& mt, float& St) {
+// base-2 statistics: student logits in rs, teacher logits in tv[OFF..OFF+31].
+// Indices stay compile-time so the values stay in registers. x = z k2 with
+// k2 = log2(e) / tau; A is kept in raw logit units (times k2 at the end).
+template <bool PARTIAL, int OFF>
+__device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint32_t (&tv)[kColsPerWarp], int nvalid,
+                                           float k2, float& ms, float& Ss, float& A, float& mt, float& St) {
   float cms = -INFINITY, cmt = -INFINITY;
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
     if (!PARTIAL || j < nvalid) {
       cms = fmaxf(cms, __uint_as_float(rs[j]));
-      cmt = fmaxf(cmt, __uint_as_float(rt[j]));
+      cmt = fmaxf(cmt, __uint_as_float(tv[OFF + j]));
     }
   }
   // k2 > 0, so the scaled maximum is the maximum of the scaled values
@@ -124,7 +143,7 @@ __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint3
   for (int j = 0; j < 32; ++j) {
     if (!PARTIAL || j < nvalid) {
       const float zs = __uint_as_float(rs[j]);
-      const float zt = __uint_as_float(rt[j]);
+      const float zt = __uint_as_float(tv[OFF + j]);
       const float e = exp2f(fmaf(zs, k2, -ms));
       Ss += e;
       A = fmaf(e, zs - zt, A);
@@ -133,40 +152,84 @@ __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint3
   }
 }
 
-template <int BN, bool BWD, int NEPI>
-__global__ void __launch_bounds__(64 + 32 * NEPI, 1)
+// Forward: 32 student columns of one row folded with the matching teacher columns.
+template <int C>
+__device__ __forceinline__ void fwd_chunk(uint32_t ts, const uint32_t (&tv)[kColsPerWarp], int nvalid_base,
+                                          float k2, float& ms, float& Ss, float& A, float& mt, float& St) {
+  uint32_t rs[32];
+  tmem_ld32(ts + C * 32, rs);
+  const int nvalid = nvalid_base - C * 32;
+  if (nvalid >= 32)
+    fold_chunk<false, C * 32>(rs, tv, 32, k2, ms, Ss, A, mt, St);
+  else if (nvalid > 0)
+    fold_chunk<true, C * 32>(rs, tv, nvalid, k2, ms, Ss, A, mt, St);
+}
+
+// Backward: dz for 32 columns of one row, packed to bf16 into this warp's
+// 128B-swizzled staging box (64 columns per box; chunk C fills half of box C/2).
+template <int C>
+__device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kColsPerWarp], float k2, float b1,
+                                          float kc, float cc, uint32_t stg, int lane) {
+  uint32_t rs[32];
+  tmem_ld32(ts + C * 32, rs);
+  uint32_t w[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    float dz2[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const float zs = __uint_as_float(rs[2 * j + e]);
+      const float zt = __uint_as_float(tv[C * 32 + 2 * j + e]);
+      const float ps = exp2f(fmaf(zs, k2, -b1));
+      dz2[e] = ps * fmaf(zs - zt, kc, -cc);
+    }
+    w[j] = pack_bf16x2(dz2[0], dz2[1]);
+  }
+  const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
+  const uint32_t jb = (uint32_t)(C & 1) * 4u;
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj)
+    st_shared_v4(box + sw128_offset((uint32_t)lane, jb + jj), w[4 * jj], w[4 * jj + 1], w[4 * jj + 2],
+                 w[4 * jj + 3]);
+}
+
+template <bool BWD, bool PAIR>
+__global__ void __launch_bounds__(kThreads, 1)
     k_fused_logits(const __grid_constant__ CUtensorMap tm_hs, const __grid_constant__ CUtensorMap tm_ht,
                    const __grid_constant__ CUtensorMap tm_ws, const __grid_constant__ CUtensorMap tm_wt,
                    const __grid_constant__ CUtensorMap tm_dz, const FusedParams p) {
-  using C = FusedCfg<BN, BWD, NEPI>;
+  using C = FusedCfg<BWD, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* stage_base = smem;
   uint8_t* staging = smem + C::kStages * C::kStageBytes;
-  float* merge = reinterpret_cast<float*>(staging + NEPI * C::kStagingPerWarp);
+  float* merge = reinterpret_cast<float*>(staging + kNEpi * C::kStagingPerWarp);
   uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(merge) + C::kMergeBytes);
   uint64_t* empty = full + C::kStages;
-  uint64_t* acc_full = empty + C::kStages;
-  uint64_t* acc_empty = acc_full + C::kBufs;
-  uint64_t* mma_done = acc_empty + C::kBufs;
-  uint64_t* merge_full = mma_done + 1;   // [4], forward with two warps per quadrant
-  uint64_t* merge_empty = merge_full + 4;  // [4]
+  uint64_t* acc_full = empty + C::kStages;  // both segments of a tile computed
+  uint64_t* t_free = acc_full + 1;          // teacher columns read by every epilogue warp
+  uint64_t* s_free = t_free + 1;            // student columns read by every epilogue warp
+  uint64_t* mma_done = s_free + 1;
+  uint64_t* merge_full = mma_done + 1;      // [4]
+  uint64_t* merge_empty = merge_full + 4;   // [4]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(merge_empty + 4);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   uint32_t* status = &p.ctrl->status;
   const uint64_t lim = p.wait_limit_ns;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;  // CTA rank within the pair
+  const int worker = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int n_workers = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int b = 0; b < C::kBufs; ++b) {
-      mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], NEPI);
-    }
+    mbar_init(acc_full, 1);
+    mbar_init(t_free, C::kFreeCount);
+    mbar_init(s_free, C::kFreeCount);
     mbar_init(mma_done, 1);
     for (int qd = 0; qd < 4; ++qd) {
       mbar_init(&merge_full[qd], 1);
@@ -182,17 +245,27 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
     if (BWD) prefetch_tmap(&tm_dz);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(tmem_slot, 512);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, 512);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync_all();  // barriers of both CTAs initialised before any remote use
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  const uint32_t tmem_t = tmem_base;        // teacher accumulator columns
+  const uint32_t tmem_s = tmem_base + kBN;  // student accumulator columns
 
   const int R = p.ctrl->R;
   FusedSchedule sch;
-  sch.init(R, p.V, BN, gridDim.x, p.group_rows, BWD);
+  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit, BWD);
   if (!BWD && blockIdx.x == 0 && threadIdx.x == 0) p.ctrl->n_vsplit = sch.n_vs;
   const int nks = (p.d_s + kKBlock - 1) / kKBlock;
   const int nkt = (p.d_t + kKBlock - 1) / kKBlock;
@@ -202,23 +275,34 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
     if (lane == 0) {
       uint32_t stage = 0, phase = 0;
       bool ok = true, any = false;
-      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x) {
+      // a pair counts both CTAs' bytes on the leader's full barriers
+      const uint32_t full_leader = PAIR ? mapa_shared(smem_u32(full), 0u) : smem_u32(full);
+      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
+        const int row0 = rt * C::kTileRows + (int)rank * kRowTile;
         for (int vt = vb; ok && vt < ve; ++vt) {
-          for (int seg = 0; ok && seg < 2; ++seg) {
-            const CUtensorMap* ta = seg ? &tm_ht : &tm_hs;
-            const CUtensorMap* tb = seg ? &tm_wt : &tm_ws;
-            const int nk = seg ? nkt : nks;
+          const int wrow0 = vt * kBN + (int)rank * C::kBRows;
+          for (int seg = 0; ok && seg < 2; ++seg) {  // teacher, then student
+            const CUtensorMap* ta = seg ? &tm_hs : &tm_ht;
+            const CUtensorMap* tb = seg ? &tm_ws : &tm_wt;
+            const int nk = seg ? nks : nkt;
             for (int kb = 0; kb < nk; ++kb) {
               if (!mbar_wait(&empty[stage], phase ^ 1u, status, lim)) {
                 ok = false;
                 break;
               }
               uint8_t* sa = stage_base + stage * C::kStageBytes;
-              mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
-              tma_load_2d(sa, ta, &full[stage], kb * kKBlock, rt * kRowTile);
-              tma_load_2d(sa + C::kABytes, tb, &full[stage], kb * kKBlock, vt * BN);
+              if (PAIR) {
+                if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * C::kStageBytes);
+                const uint32_t fb = full_leader + stage * 8u;
+                tma_load_2d_pair(sa, ta, fb, kb * kKBlock, row0);
+                tma_load_2d_pair(sa + C::kABytes, tb, fb, kb * kKBlock, wrow0);
+              } else {
+                mbar_arrive_expect_tx(&full[stage], C::kStageBytes);
+                tma_load_2d(sa, ta, &full[stage], kb * kKBlock, row0);
+                tma_load_2d(sa + C::kABytes, tb, &full[stage], kb * kKBlock, wrow0);
+              }
               any = true;
               if (++stage == (uint32_t)C::kStages) {
                 stage = 0;
@@ -228,8 +312,9 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
           }
         }
       }
-      if (!ok && any) {
-        // Let every copy already issued land before the CTA can exit.
+      if (!ok && any && rank == 0) {
+        // Let every copy already issued land before the CTA can exit (in a pair,
+        // the leader's barriers also count the peer's copies).
         for (int s = 0; s < C::kStages; ++s) {
           const uint32_t par = ((uint32_t)s < stage) ? phase : (phase ^ 1u);
           mbar_wait_drain(&full[s], par, lim);
@@ -238,25 +323,24 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kRowTile, BN, false, false);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(C::kTileRows, kBN, false, false);
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x) {
+      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
         for (int vt = vb; ok && vt < ve; ++vt, ++lt) {
-          const int buf = lt % C::kBufs;
-          const uint32_t acc_par = (uint32_t)(lt / C::kBufs) & 1u;
-          if (!mbar_wait(&acc_empty[buf], acc_par ^ 1u, status, lim)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
+          const uint32_t free_par = ((uint32_t)lt & 1u) ^ 1u;  // previous tile's release
           for (int seg = 0; ok && seg < 2; ++seg) {
-            const uint32_t d_tmem = tmem_base + (uint32_t)((buf * 2 + seg) * BN);
-            const int nk = seg ? nkt : nks;
+            if (!mbar_wait(seg ? s_free : t_free, free_par, status, lim)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = seg ? tmem_s : tmem_t;
+            const int nk = seg ? nks : nkt;
             for (int kb = 0; kb < nk; ++kb) {
               if (!mbar_wait(&full[stage], phase, status, lim)) {
                 ok = false;
@@ -267,38 +351,57 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
               const uint32_t sb = sa + C::kABytes;
 #pragma unroll
               for (int k = 0; k < kKBlock / 16; ++k) {
-                umma_bf16(d_tmem, sdesc_sw128(sa + k * 32, 16, 1024), sdesc_sw128(sb + k * 32, 16, 1024), idesc,
-                          (kb | k) != 0);
+                const uint64_t ad = sdesc_sw128(sa + k * 32, 16, 1024);
+                const uint64_t bd = sdesc_sw128(sb + k * 32, 16, 1024);
+                if (PAIR)
+                  umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | k) != 0);
+                else
+                  umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0);
               }
-              umma_commit(&empty[stage]);
+              if (PAIR)
+                umma_commit_pair_mc(&empty[stage], 0x3);
+              else
+                umma_commit(&empty[stage]);
               if (++stage == (uint32_t)C::kStages) {
                 stage = 0;
                 phase ^= 1u;
               }
             }
           }
-          if (ok) umma_commit(&acc_full[buf]);
+          if (ok) {
+            if (PAIR)
+              umma_commit_pair_mc(acc_full, 0x3);
+            else
+              umma_commit(acc_full);
+          }
         }
       }
       // Every MMA issued by this thread completes before TMEM is released.
-      umma_commit(mma_done);
+      if (PAIR)
+        umma_commit_pair_mc(mma_done, 0x1);
+      else
+        umma_commit(mma_done);
       mbar_wait_drain(mma_done, 0, lim);
     }
   } else {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - 2;                 // epilogue warp index
     const int q = warp & 3;                  // TMEM lane quadrant this warp may access
-    const int half = ew / 4;                 // which share of the tile's columns
-    const int cbase = half * C::kColsPerWarp;
+    const int half = ew / 4;                 // which 128 of the tile's 256 columns
+    const int cbase = half * kColsPerWarp;
     const int row_in_tile = q * 32 + lane;
     const uint32_t t_lane = (uint32_t)(q * 32) << 16;
+    // the MMA issuer (in the pair's leader) waits for every epilogue warp of the pair
+    const uint32_t t_free_addr = PAIR ? mapa_shared(smem_u32(t_free), 0u) : smem_u32(t_free);
+    const uint32_t s_free_addr = PAIR ? mapa_shared(smem_u32(s_free), 0u) : smem_u32(s_free);
     int lt = 0, nu = 0;
     bool ok = true;
-    uint8_t* stg = staging + ew * C::kStagingPerWarp;
-    for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x, ++nu) {
+    const uint32_t stg = smem_u32(staging + ew * C::kStagingPerWarp);
+    for (int u = worker; ok && u < sch.n_units; u += n_workers, ++nu) {
       int rt, split, vb, ve;
       sch.unit(u, rt, split, vb, ve);
-      const int row = rt * kRowTile + row_in_tile;
+      const int row_base = rt * C::kTileRows + (int)rank * kRowTile;
+      const int row = row_base + row_in_tile;
       float ms = -INFINITY, Ss = 0.f, A = 0.f, mt = -INFINITY, St = 0.f;
       // backward row constants: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc)
       float b1 = 0.f, kc = 0.f, cc = 0.f;
@@ -309,103 +412,99 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
         cc = rc.z * rc.y;
       }
       for (int vt = vb; vt < ve; ++vt, ++lt) {
-        const int buf = lt % C::kBufs;
-        const uint32_t acc_par = (uint32_t)(lt / C::kBufs) & 1u;
         // warp-uniform outcome: the TMEM loads below are .sync.aligned
-        if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[buf], acc_par, status, lim))) {
+        if (!__all_sync(0xffffffffu, mbar_wait(acc_full, (uint32_t)lt & 1u, status, lim))) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const int col0 = vt * BN + cbase;
-        const uint32_t ts = tmem_base + t_lane + (uint32_t)(buf * 2 * BN + cbase);
-        const uint32_t tt = ts + BN;
-#pragma unroll 1
-        for (int c = 0; c < C::kColsPerWarp / 32; ++c) {
-          uint32_t rs[32], rtt[32];
-          tmem_ld32x2(ts + c * 32, tt + c * 32, rs, rtt);
-          if (!BWD) {
-            const int nvalid = p.V - (col0 + c * 32);
-            if (nvalid >= 32)
-              fold_chunk<false>(rs, rtt, 32, p.k2, ms, Ss, A, mt, St);
-            else if (nvalid > 0)
-              fold_chunk<true>(rs, rtt, nvalid, p.k2, ms, Ss, A, mt, St);
-          } else {
-            const int h = c >> 1;  // 64-column box of this warp's staging tile
-            if ((c & 1) == 0) {
-              if (lane == 0) bulk_wait_read<C::kColsPerWarp / 64 - 1>();
-              __syncwarp();
-            }
-            uint32_t w[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              float dz2[2];
-#pragma unroll
-              for (int e = 0; e < 2; ++e) {
-                const float zs = __uint_as_float(rs[2 * j + e]);
-                const float zt = __uint_as_float(rtt[2 * j + e]);
-                const float ps = exp2f(fmaf(zs, p.k2, -b1));
-                dz2[e] = ps * fmaf(zs - zt, kc, -cc);
-              }
-              w[j] = pack_bf16x2(dz2[0], dz2[1]);
-            }
-            const uint32_t box = smem_u32(stg + h * 4096);
-            const uint32_t jb = (uint32_t)(c & 1) * 4u;
-#pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-              st_shared_v4(box + sw128_offset((uint32_t)lane, jb + jj), w[4 * jj], w[4 * jj + 1], w[4 * jj + 2],
-                           w[4 * jj + 3]);
-            }
-            if (c & 1) {
-              fence_proxy_async_smem();
-              __syncwarp();
-              if (lane == 0) {
-                tma_store_2d(&tm_dz, stg + h * 4096, col0 + h * 64, rt * kRowTile + q * 32);
-                bulk_commit();
-              }
-            }
+        // teacher columns to registers, then release them to the next tile's MMAs
+        uint32_t tv[kColsPerWarp];
+        tmem_ld128(tmem_t + t_lane + (uint32_t)cbase, tv);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (PAIR)
+            mbar_arrive_cluster(t_free_addr);
+          else
+            mbar_arrive(t_free);
+        }
+        const int col0 = vt * kBN + cbase;
+        const uint32_t ts = tmem_s + t_lane + (uint32_t)cbase;
+        if (!BWD) {
+          const int nv = p.V - col0;
+          fwd_chunk<0>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+          fwd_chunk<1>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+          fwd_chunk<2>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+          fwd_chunk<3>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+        } else {
+          // staging box h of this warp is rewritten only after its previous TMA
+          // store has finished reading it
+          if (lane == 0) bulk_wait_read<1>();
+          __syncwarp();
+          bwd_chunk<0>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+          bwd_chunk<1>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, row_base + q * 32);
+            bulk_commit();
+            bulk_wait_read<1>();
+          }
+          __syncwarp();
+          bwd_chunk<2>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+          bwd_chunk<3>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, row_base + q * 32);
+            bulk_commit();
           }
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        if (lane == 0) {
+          if (PAIR)
+            mbar_arrive_cluster(s_free_addr);
+          else
+            mbar_arrive(s_free);
+        }
       }
       if (!BWD && ok) {
         A *= p.k2;  // A was accumulated in raw logit units
-        if (C::kHalves > 1) {
-          // the two warps of a quadrant fold their column shares: half 1 hands its
-          // statistics to half 0 through shared memory
-          float* mb = merge + q * 5 * 32;
-          if (half == 1) {
-            if (nu > 0 && !__all_sync(0xffffffffu, mbar_wait(&merge_empty[q], (uint32_t)(nu - 1) & 1u, status, lim))) {
-              ok = false;
-              break;
-            }
-            mb[0 * 32 + lane] = ms;
-            mb[1 * 32 + lane] = Ss;
-            mb[2 * 32 + lane] = A;
-            mb[3 * 32 + lane] = mt;
-            mb[4 * 32 + lane] = St;
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&merge_full[q]);
-            continue;
-          }
-          if (!__all_sync(0xffffffffu, mbar_wait(&merge_full[q], (uint32_t)nu & 1u, status, lim))) {
+        // the two warps of a quadrant fold their column shares: half 1 hands its
+        // statistics to half 0 through shared memory
+        float* mb = merge + q * 5 * 32;
+        if (half == 1) {
+          if (nu > 0 &&
+              !__all_sync(0xffffffffu, mbar_wait(&merge_empty[q], (uint32_t)(nu - 1) & 1u, status, lim))) {
             ok = false;
             break;
           }
-          const float ms1 = mb[0 * 32 + lane], Ss1 = mb[1 * 32 + lane], A1 = mb[2 * 32 + lane];
-          const float mt1 = mb[3 * 32 + lane], St1 = mb[4 * 32 + lane];
+          mb[0 * 32 + lane] = ms;
+          mb[1 * 32 + lane] = Ss;
+          mb[2 * 32 + lane] = A;
+          mb[3 * 32 + lane] = mt;
+          mb[4 * 32 + lane] = St;
           __syncwarp();
-          if (lane == 0) mbar_arrive(&merge_empty[q]);
-          const float Ms = fmaxf(ms, ms1), Mt = fmaxf(mt, mt1);
-          const float f0 = exp2f(ms - Ms), f1 = exp2f(ms1 - Ms);
-          Ss = Ss * f0 + Ss1 * f1;
-          A = A * f0 + A1 * f1;
-          St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
-          ms = Ms;
-          mt = Mt;
+          if (lane == 0) mbar_arrive(&merge_full[q]);
+          continue;
         }
+        if (!__all_sync(0xffffffffu, mbar_wait(&merge_full[q], (uint32_t)nu & 1u, status, lim))) {
+          ok = false;
+          break;
+        }
+        const float ms1 = mb[0 * 32 + lane], Ss1 = mb[1 * 32 + lane], A1 = mb[2 * 32 + lane];
+        const float mt1 = mb[3 * 32 + lane], St1 = mb[4 * 32 + lane];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&merge_empty[q]);
+        const float Ms = fmaxf(ms, ms1), Mt = fmaxf(mt, mt1);
+        const float f0 = exp2f(ms - Ms), f1 = exp2f(ms1 - Ms);
+        Ss = Ss * f0 + Ss1 * f1;
+        A = A * f0 + A1 * f1;
+        St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
+        ms = Ms;
+        mt = Mt;
         const size_t plane = (size_t)p.T_pad;
         float* base = p.partials + (size_t)split * 5 * plane + row;
         base[0 * plane] = ms;
@@ -419,33 +518,63 @@ __global__ void __launch_bounds__(64 + 32 * NEPI, 1)
   }
 
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync_all();  // the pair's MMAs and both epilogues are done with TMEM
+  else
+    __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    if (PAIR)
+      tmem_dealloc_pair(tmem_base, 512);
+    else
+      tmem_dealloc(tmem_base, 512);
   }
 }
 
-template <int BN, bool BWD, int NEPI>
+template <bool BWD, bool PAIR>
 cudaError_t launch_fused_impl(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                               const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
                               cudaStream_t s) {
-  using C = FusedCfg<BN, BWD, NEPI>;
+  using C = FusedCfg<BWD, PAIR>;
   static_assert(C::kSmem <= 232448, "shared memory budget");
-  auto kern = k_fused_logits<BN, BWD, NEPI>;
+  auto kern = k_fused_logits<BWD, PAIR>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, C::kThreads, C::kSmem, s>>>(hs, ht, ws, wt, dz, p);
+  if (!PAIR) {
+    kern<<<grid, kThreads, C::kSmem, s>>>(hs, ht, ws, wt, dz, p);
+    return cudaGetLastError();
+  }
+  // One CTA pair per two SMs, no more pairs than can be resident at once.
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3((unsigned)(grid & ~1), 1, 1);
+  int max_clusters = 0;
+  e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+  if (e != cudaSuccess) return e;
+  if (max_clusters < 1) return cudaErrorInvalidConfiguration;
+  const int pairs = (grid / 2) < max_clusters ? (grid / 2) : max_clusters;
+  cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
+  e = cudaLaunchKernelEx(&cfg, kern, hs, ht, ws, wt, dz, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 template <bool BWD>
-cudaError_t launch_fused_bn(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
-                            const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
-                            cudaStream_t s) {
-  switch (fused_bn(p)) {
-    case 128: return launch_fused_impl<128, BWD, 4>(hs, ht, ws, wt, dz, p, grid, s);
-    case 256: return launch_fused_impl<256, BWD, 8>(hs, ht, ws, wt, dz, p, grid, s);
+cudaError_t launch_fused_mode(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
+                              const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
+                              cudaStream_t s) {
+  switch (fused_mode(p)) {
+    case kFusedBN256: return launch_fused_impl<BWD, false>(hs, ht, ws, wt, dz, p, grid, s);
+    case kFusedPair256: return launch_fused_impl<BWD, true>(hs, ht, ws, wt, dz, p, grid, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -454,13 +583,13 @@ cudaError_t launch_fused_bn(const CUtensorMap& hs, const CUtensorMap& ht, const 
 
 cudaError_t launch_fused_forward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                  const CUtensorMap& wt, const FusedParams& p, int grid, cudaStream_t s) {
-  return launch_fused_bn<false>(hs, ht, ws, wt, hs, p, grid, s);
+  return launch_fused_mode<false>(hs, ht, ws, wt, hs, p, grid, s);
 }
 
 cudaError_t launch_fused_backward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                   const CUtensorMap& wt, const CUtensorMap& dz_store, const FusedParams& p,
                                   int grid, cudaStream_t s) {
-  return launch_fused_bn<true>(hs, ht, ws, wt, dz_store, p, grid, s);
+  return launch_fused_mode<true>(hs, ht, ws, wt, dz_store, p, grid, s);
 }
 
 }  // namespace opd

@@ -13,27 +13,34 @@ struct Ctrl;
 // Tile geometry shared by host and device code.
 constexpr int kRowTile = 128;   // token rows per MMA tile (TMEM lanes)
 constexpr int kKBlock = 64;     // bf16 elements per 128-byte swizzled row
-constexpr int kMaxVSplit = 64;  // vocabulary splits of the forward statistics
+constexpr int kMaxVSplit = 128; // vocabulary splits of the forward statistics (partials planes)
 constexpr int kMaxKSplit = 16;  // K splits of the dH_s GEMM
-constexpr int kFusedBN = 256;   // default vocabulary columns per fused tile (128 or 256)
+constexpr int kRowPad = 256;    // gathered rows are zero-padded to a multiple of this
 constexpr int kGemmBN = 256;    // output columns per gradient-GEMM tile
+
+// Fused-kernel tilings: 128 x 256 tiles on one CTA, or 256 x 256 tiles on a CTA
+// pair (tcgen05 cta_group::2).
+enum FusedMode : int32_t { kFusedDefault = 0, kFusedBN256 = 2, kFusedPair256 = 3 };
+constexpr FusedMode kFusedDefaultMode = kFusedPair256;
+
+// Rows of W (vocabulary entries) one CTA stages per tile: the W tensor maps' box height.
+constexpr int fused_w_box(int mode) { return mode == kFusedBN256 ? 256 : 128; }
 
 struct FusedParams {
   Ctrl* ctrl;
   int32_t V, d_s, d_t;
-  int32_t T_pad;        // rows of the gathered buffers (multiple of kRowTile)
+  int32_t T_pad;        // rows of the gathered buffers (multiple of kRowPad)
   int32_t group_rows;   // row tiles walked together (L2 raster group)
   float k2;             // log2(e) / tau
   float inv_tau;
   uint64_t wait_limit_ns;
-  float* partials;      // forward: [kMaxVSplit][5][T_pad]
+  float* partials;      // forward: [max_vsplit][5][T_pad]
+  int32_t max_vsplit;   // vocabulary splits the forward may use (<= kMaxVSplit; sizes partials)
   const float4* rowc;   // backward: [T_pad] = (lse_s log2 e, lse_s - lse_t + KL, g / tau, 0)
-  int32_t bn;           // vocabulary columns per tile: 128 or 256 (0 = kFusedBN); the W tensor
-                        // maps must use the same box height
+  int32_t mode;         // FusedMode; the W tensor maps' box height must be fused_w_box(mode)
 };
 
-// Tile width the fused kernels use for these parameters.
-inline int fused_bn(const FusedParams& p) { return p.bn == 0 ? kFusedBN : p.bn; }
+inline int fused_mode(const FusedParams& p) { return p.mode == kFusedDefault ? kFusedDefaultMode : p.mode; }
 
 struct GemmParams {
   Ctrl* ctrl;

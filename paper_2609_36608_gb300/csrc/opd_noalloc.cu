@@ -31,10 +31,11 @@ namespace {
 constexpr int kMaxRows = OPD_KL_NOALLOC_MAX_ROWS;                          // token rows per call
 constexpr size_t kCtrlBytes = 256;                                         // Ctrl block
 constexpr size_t kPosBytes = (size_t)kMaxRows * 4;                         // pos[T]
-constexpr size_t kPartialBytes = (size_t)kMaxVSplit * 5 * kMaxRows * 4;    // [split][5][row] floats
+constexpr int kSplits = 64;                                                 // vocabulary splits used here
+constexpr size_t kPartialBytes = (size_t)kSplits * 5 * kMaxRows * 4;       // [split][5][row] floats
 constexpr size_t kScratchBytes = kCtrlBytes + kPosBytes + kPartialBytes;  // 5,259,520 bytes
 static_assert(sizeof(Ctrl) <= kCtrlBytes, "control block");
-static_assert(kMaxRows % kRowTile == 0, "row cap is a whole number of row tiles");
+static_assert(kMaxRows % kRowPad == 0, "row cap is a whole number of padded row tiles");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
@@ -124,13 +125,13 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   float* partials = reinterpret_cast<float*>(base + kCtrlBytes + kPosBytes);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const int32_t T = (int32_t)p.T;
-  const int32_t T_pad = (T + kRowTile - 1) / kRowTile * kRowTile;
+  const int32_t T_pad = (T + kRowPad - 1) / kRowPad * kRowPad;
 
   CUtensorMap hs, ht, ws, wt;
   if (!tmap_bf16(&hs, H_s, (uint64_t)p.d_s, (uint64_t)T, kKBlock, kRowTile) ||
       !tmap_bf16(&ht, H_t, (uint64_t)p.d_t, (uint64_t)T, kKBlock, kRowTile) ||
-      !tmap_bf16(&ws, W_s, (uint64_t)p.d_s, (uint64_t)p.V, kKBlock, kFusedBN) ||
-      !tmap_bf16(&wt, W_t, (uint64_t)p.d_t, (uint64_t)p.V, kKBlock, kFusedBN))
+      !tmap_bf16(&ws, W_s, (uint64_t)p.d_s, (uint64_t)p.V, kKBlock, fused_w_box(kFusedDefaultMode)) ||
+      !tmap_bf16(&wt, W_t, (uint64_t)p.d_t, (uint64_t)p.V, kKBlock, fused_w_box(kFusedDefaultMode)))
     return OPD_ERR_CUDA;
 
   k_noalloc_rows<<<1, 1024, 0, s>>>(mask, T);
@@ -147,6 +148,7 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.inv_tau = 1.0f / p.temperature;
   fp.wait_limit_ns = 2000000000ull;
   fp.partials = partials;
+  fp.max_vsplit = kSplits;
   fp.rowc = nullptr;
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
   if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, sms, s) != cudaSuccess) return OPD_ERR_CUDA;

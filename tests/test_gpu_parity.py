@@ -103,10 +103,11 @@ def _small_bf16(**kw):
     return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
 
 
-@pytest.fixture(params=[128, 256], ids=["bn128", "bn256"])
+@pytest.fixture(params=["bn256", "pair256"])
 def fused_bn(request, monkeypatch):
-    """Both vocabulary tile widths of the fused kernels (the library reads the override per call)."""
-    monkeypatch.setenv("OPD_KL_FUSED_BN", str(request.param))
+    """Every tiling of the fused kernels: 128 x 256 tiles on one CTA, 256 x 256 tiles on a CTA pair
+    (the library reads the override on every call)."""
+    monkeypatch.setenv("OPD_KL_FUSED", request.param)
     return request.param
 
 
