@@ -55,6 +55,14 @@ def _load():
         lib.opd_oracle_kl.restype = ctypes.c_int
         lib.opd_oracle_seq_mean_token_mean_weights.argtypes = [p, p, i64, ctypes.c_double, p]
         lib.opd_oracle_seq_mean_token_mean_weights.restype = ctypes.c_int
+        dbl = ctypes.c_double
+        lib.opd_oracle_score.argtypes = [i64, i64, i64, dbl, ctypes.c_int, p, p, p, p, i64, p, p, ctypes.c_int]
+        lib.opd_oracle_score.restype = ctypes.c_int
+        lib.opd_oracle_surrogate.argtypes = [i64, i64, i64, dbl, ctypes.c_int, p, p, p, p, p, p, p, dbl, dbl, dbl,
+                                             p, i64, p, p, p, p, p, p, ctypes.c_int]
+        lib.opd_oracle_surrogate.restype = ctypes.c_int
+        lib.opd_oracle_dual_clip.argtypes = [i64, p, p, p, dbl, dbl, dbl, p, p]
+        lib.opd_oracle_dual_clip.restype = ctypes.c_int
         _lib = lib
     return _lib
 
@@ -135,3 +143,92 @@ def seq_mean_token_mean_weights(seg_id, mask, eps: float = 1e-8) -> np.ndarray:
     if rc != 0:
         raise ValueError("oracle rejected its arguments")
     return w
+
+
+# Constants of the surrogate (Appendix B.4): clipping width, dual-clip constant, log-ratio clip.
+DELTA = 0.2
+KAPPA = 3.0
+LOG_RATIO_CLIP = 20.0
+
+
+def score(H, W, tokens, tau: float = 1.0, rows=None, n_threads: Optional[int] = None):
+    """(lse, logp) of the given tokens under one head, float64, for every listed row."""
+    lib = _load()
+    Hh, kind = _as_input(H)
+    Wh, k2 = _as_input(W)
+    if kind != k2:
+        raise ValueError("H and W must share one element kind")
+    T, d = Hh.shape
+    V = Wh.shape[0]
+    if Wh.shape != (V, d):
+        raise ValueError("shape mismatch")
+    tok = np.ascontiguousarray(tokens, dtype=np.int32)
+    r = None if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    n = T if r is None else r.shape[0]
+    lse = np.zeros(n)
+    logp = np.zeros(n)
+    rc = lib.opd_oracle_score(T, d, V, float(tau), kind, _ptr(Hh), _ptr(Wh), _ptr(tok), _ptr(r), n, _ptr(lse),
+                              _ptr(logp), int(n_threads or default_threads()))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return lse, logp
+
+
+@dataclass
+class SurrogateResult:
+    loss: np.ndarray
+    logp_s: np.ndarray
+    adv: np.ndarray
+    dZ: Optional[np.ndarray]
+    dH_s: Optional[np.ndarray]
+    dW_s: Optional[np.ndarray]
+
+
+def surrogate(H_s, W_s, tokens, logp_old, logp_teacher, mask, w, tau: float = 1.0, delta: float = DELTA,
+              kappa: float = KAPPA, clip: float = LOG_RATIO_CLIP, rows=None, want_dZ: bool = False,
+              want_dH: bool = True, want_dW: bool = True, n_threads: Optional[int] = None) -> SurrogateResult:
+    """Sampled-token dual-clip surrogate (student side) and its gradient, float64."""
+    lib = _load()
+    Hh, kind = _as_input(H_s)
+    Wh, k2 = _as_input(W_s)
+    if kind != k2:
+        raise ValueError("H_s and W_s must share one element kind")
+    T, d = Hh.shape
+    V = Wh.shape[0]
+    if Wh.shape != (V, d):
+        raise ValueError("shape mismatch")
+    tok = np.ascontiguousarray(tokens, dtype=np.int32)
+    lo = np.ascontiguousarray(logp_old, dtype=np.float64)
+    lt = np.ascontiguousarray(logp_teacher, dtype=np.float64)
+    m = np.ascontiguousarray(np.asarray(mask) != 0, dtype=np.uint8)
+    ww = np.ascontiguousarray(w, dtype=np.float64)
+    for a in (tok, lo, lt, m, ww):
+        if a.shape != (T,):
+            raise ValueError("per-token inputs must have shape [T]")
+    r = None if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    n = T if r is None else r.shape[0]
+    loss, lps, adv = np.zeros(n), np.zeros(n), np.zeros(n)
+    dZ = np.zeros((n, V)) if want_dZ else None
+    dH = np.zeros((n, d)) if want_dH else None
+    dW = np.zeros((V, d)) if want_dW else None
+    rc = lib.opd_oracle_surrogate(T, d, V, float(tau), kind, _ptr(Hh), _ptr(Wh), _ptr(tok), _ptr(lo), _ptr(lt),
+                                  _ptr(m), _ptr(ww), float(delta), float(kappa), float(clip), _ptr(r), n,
+                                  _ptr(loss), _ptr(lps), _ptr(adv), _ptr(dZ), _ptr(dH), _ptr(dW),
+                                  int(n_threads or default_threads()))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return SurrogateResult(loss, lps, adv, dZ, dH, dW)
+
+
+def dual_clip(logp_s, logp_old, A, delta: float = DELTA, kappa: float = KAPPA, clip: float = LOG_RATIO_CLIP):
+    """Per-token dual-clip loss and d loss / d logp_s (elementwise)."""
+    lib = _load()
+    a = np.ascontiguousarray(logp_s, dtype=np.float64)
+    b = np.ascontiguousarray(logp_old, dtype=np.float64)
+    c = np.ascontiguousarray(A, dtype=np.float64)
+    loss, dl = np.zeros(a.shape[0]), np.zeros(a.shape[0])
+    rc = lib.opd_oracle_dual_clip(a.shape[0], _ptr(a), _ptr(b), _ptr(c), float(delta), float(kappa), float(clip),
+                                  _ptr(loss), _ptr(dl))
+    if rc != 0:
+        raise ValueError("oracle rejected its arguments")
+    return loss, dl

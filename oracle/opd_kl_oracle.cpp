@@ -20,6 +20,16 @@
 //   dW_s[k,:] = sum_i dz_i[k] H_s[i,:]
 //   masked rows (mask[i] == 0): KL_i = 0, dz = 0, dH_s[i,:] = 0, no dW_s term.
 //
+// Also, for the sampled-token surrogate the paper optimises (Appendix B.4,
+// Eq. opd-token-advantage, opd-ratio, opd-dual-clip, opd-surrogate):
+//   log pi(x_i) = u[x_i] - logsumexp(u)                 token scoring under one head
+//   A_i = sg[ log pi_teacher(x_i) - log pi_old(x_i) ]    (0 on masked rows)
+//   rho_i = exp(clip(log pi_student(x_i) - log pi_old(x_i), -c, c))      c = 20
+//   l_clip = -min(rho A, clip(rho, 1 - delta, 1 + delta) A)             delta = 0.2
+//   l_DC = min(l_clip, -kappa A) if A < 0 else l_clip                   kappa = 3
+//   L = sum_i w_i l_DC,i with w the seq-mean-token-mean weights
+//   dL/dz_s[i,k] = w_i dl/drho drho/dr (1/tau) (1[k = x_i] - p_s[i,k])
+//
 // Everything is plain: logits are materialised, sums run in index order with
 // one double accumulator, no blocking, no online rescaling. Threads only split
 // independent rows (phase 1) or independent vocab rows of dW_s (phase 2).
@@ -212,6 +222,155 @@ int opd_oracle_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t*
     }
     w_out[i] = 1.0 / (n_responses * (supervised[seg_id[i]] + eps));
   }
+  return 0;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Token scoring and the sampled-token surrogate (Appendix B.4).
+// ---------------------------------------------------------------------------
+
+namespace {
+
+// Per-token dual-clip PPO loss and its derivative with respect to the student
+// log-probability of the sampled token (the advantage A is a constant: stop-gradient).
+//   r = logp_s - logp_old; rho = exp(clip(r, -c, c)); drho/dr = rho inside (-c, c), else 0
+//   l_clip = -min(rho A, clip(rho, 1-delta, 1+delta) A); the unclipped product is the
+//   active branch when rho A <= clip(rho) A, otherwise the clipped one (zero slope).
+//   l_DC = min(l_clip, -kappa A) when A < 0; l_clip is active when l_clip <= -kappa A.
+void dual_clip_loss(double logp_s, double logp_old, double A, double delta, double kappa, double c,
+                    double* loss, double* dloss_dlogp) {
+  const double r = logp_s - logp_old;
+  const double rc = r < -c ? -c : (r > c ? c : r);
+  const double rho = std::exp(rc);
+  const double drho = (r > -c && r < c) ? rho : 0.0;
+  const double lo = 1.0 - delta, hi = 1.0 + delta;
+  const double rho_clipped = rho < lo ? lo : (rho > hi ? hi : rho);
+  const double m_unclipped = rho * A;
+  const double m_clipped = rho_clipped * A;
+  double l_clip, dl_drho;
+  if (m_unclipped <= m_clipped) {
+    l_clip = -m_unclipped;
+    dl_drho = -A;
+  } else {
+    l_clip = -m_clipped;
+    dl_drho = (rho > lo && rho < hi) ? -A : 0.0;
+  }
+  double l = l_clip;
+  if (A < 0.0) {
+    const double floor_value = -kappa * A;
+    if (l_clip > floor_value) {
+      l = floor_value;
+      dl_drho = 0.0;
+    }
+  }
+  *loss = l;
+  *dloss_dlogp = dl_drho * drho;
+}
+
+}  // namespace
+
+extern "C" {
+
+// Scoring under one head for the listed rows (rows == nullptr: all T):
+//   lse[n] = logsumexp_k (H[i,:] . W[k,:]) / tau,  logp[n] = (H[i,:] . W[tokens[i],:]) / tau - lse[n]
+// Every listed row is scored, whatever its mask. Returns 0, or -1 on invalid arguments.
+int opd_oracle_score(int64_t T, int64_t d, int64_t V, double tau, int kind, const void* H, const void* W,
+                     const int32_t* tokens, const int64_t* rows, int64_t n_rows, double* lse, double* logp,
+                     int n_threads) {
+  if (T < 0 || d <= 0 || V <= 0 || !(tau > 0.0) || (kind != KIND_F32 && kind != KIND_BF16)) return -1;
+  if (!H || !W || !tokens || !lse || !logp) return -1;
+  if (!rows) n_rows = T;
+  for (int64_t n = 0; n < n_rows; ++n) {
+    const int64_t i = rows ? rows[n] : n;
+    if (i < 0 || i >= T || tokens[i] < 0 || tokens[i] >= V) return -1;
+  }
+  parallel_for(n_rows, n_threads, [&](int64_t n) {
+    const int64_t i = rows ? rows[n] : n;
+    std::vector<double> z(V);
+    logits(H, W, kind, i, d, V, z);
+    for (int64_t k = 0; k < V; ++k) z[k] /= tau;
+    lse[n] = logsumexp(z);
+    logp[n] = z[tokens[i]] - lse[n];
+  });
+  return 0;
+}
+
+// Sampled-token surrogate, student side, for the listed rows (rows == nullptr: all T).
+// Inputs per token row i: tokens[i] (sampled token), logp_old[i] (behaviour policy),
+// logp_teacher[i] (frozen teacher), mask[i], w[i] (upstream weight of l_DC,i, e.g. the
+// seq-mean-token-mean weights), constants delta, kappa and the log-ratio clip c.
+// Outputs by list position: loss[n] = l_DC (0 on masked rows), logp_s[n], adv[n] = A,
+// dZ[n, V] (optional), dH_s[n, d] (optional); dW_s[V, d] sums the listed rows (optional).
+// Returns 0, or -1 on invalid arguments.
+int opd_oracle_surrogate(int64_t T, int64_t d, int64_t V, double tau, int kind, const void* H_s, const void* W_s,
+                         const int32_t* tokens, const double* logp_old, const double* logp_teacher,
+                         const uint8_t* mask, const double* w, double delta, double kappa, double clip,
+                         const int64_t* rows, int64_t n_rows, double* loss, double* logp_s, double* adv,
+                         double* dZ, double* dH_s, double* dW_s, int n_threads) {
+  if (T < 0 || d <= 0 || V <= 0 || !(tau > 0.0) || (kind != KIND_F32 && kind != KIND_BF16)) return -1;
+  if (!H_s || !W_s || !tokens || !logp_old || !logp_teacher || !mask || !w || !loss || !logp_s || !adv)
+    return -1;
+  if (!rows) n_rows = T;
+  for (int64_t n = 0; n < n_rows; ++n) {
+    const int64_t i = rows ? rows[n] : n;
+    if (i < 0 || i >= T || tokens[i] < 0 || tokens[i] >= V) return -1;
+  }
+  const bool want_dz = dZ != nullptr || dW_s != nullptr;
+  std::vector<double> dz_all(want_dz ? static_cast<size_t>(n_rows * V) : 0);
+
+  parallel_for(n_rows, n_threads, [&](int64_t n) {
+    const int64_t i = rows ? rows[n] : n;
+    std::vector<double> z(V), dz_local(want_dz ? 0 : V);
+    double* dz = want_dz ? &dz_all[n * V] : dz_local.data();
+    logits(H_s, W_s, kind, i, d, V, z);
+    for (int64_t k = 0; k < V; ++k) z[k] /= tau;
+    const double lse = logsumexp(z);
+    const double lp = z[tokens[i]] - lse;
+    logp_s[n] = lp;
+    const bool supervised = mask[i] != 0;
+    const double A = supervised ? logp_teacher[i] - logp_old[i] : 0.0;
+    adv[n] = A;
+    double l = 0.0, dl = 0.0;
+    if (supervised) dual_clip_loss(lp, logp_old[i], A, delta, kappa, clip, &l, &dl);
+    loss[n] = l;
+    const double coef = supervised ? w[i] * dl / tau : 0.0;
+    for (int64_t k = 0; k < V; ++k) {
+      const double p = std::exp(z[k] - lse);
+      dz[k] = coef * ((k == tokens[i] ? 1.0 : 0.0) - p);
+    }
+    if (dH_s) {
+      for (int64_t j = 0; j < d; ++j) {
+        double acc = 0.0;
+        for (int64_t k = 0; k < V; ++k) acc += dz[k] * load(W_s, kind, k * d + j);
+        dH_s[n * d + j] = acc;
+      }
+    }
+  });
+  if (dZ) std::memcpy(dZ, dz_all.data(), sizeof(double) * n_rows * V);
+  if (dW_s) {
+    parallel_for(V, n_threads, [&](int64_t k) {
+      for (int64_t j = 0; j < d; ++j) {
+        double acc = 0.0;
+        for (int64_t n = 0; n < n_rows; ++n) {
+          const int64_t i = rows ? rows[n] : n;
+          acc += dz_all[n * V + k] * load(H_s, kind, i * d + j);
+        }
+        dW_s[k * d + j] = acc;
+      }
+    });
+  }
+  return 0;
+}
+
+// The per-token dual-clip loss and its slope with respect to logp_s, element by element,
+// for direct checks of the piecewise definition.
+int opd_oracle_dual_clip(int64_t n, const double* logp_s, const double* logp_old, const double* A, double delta,
+                         double kappa, double clip, double* loss, double* dloss_dlogp) {
+  if (n < 0 || (n > 0 && (!logp_s || !logp_old || !A || !loss || !dloss_dlogp))) return -1;
+  for (int64_t i = 0; i < n; ++i) dual_clip_loss(logp_s[i], logp_old[i], A[i], delta, kappa, clip, &loss[i],
+                                                 &dloss_dlogp[i]);
   return 0;
 }
 
