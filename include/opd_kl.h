@@ -103,6 +103,47 @@ opd_status opd_kl_fwd_bwd(const opd_problem* problem, const void* H_s, const voi
                           float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
                           void* stream);
 
+/* Token scoring under one head (the frozen teacher's scores, or the student's):
+ * for every row with mask[i] = 1,
+ *   lse_out[i]  = logsumexp_v (H[i,:] . W[v,:]) / temperature
+ *   logp_out[i] = (H[i,:] . W[tokens[i],:]) / temperature - lse_out[i]
+ * (zeros on rows with mask 0). ActFirst-OPD Appendix B.4: the teacher's log-probability
+ * of each generated token enters the token advantage (Eq. opd-token-advantage), the
+ * student's enters the ratio (Eq. opd-ratio). H [T, d], W [V, d] bf16 with d =
+ * problem->d_s (problem->d_t is not used; pass any valid value, e.g. d_s); tokens [T]
+ * int32 in [0, V) (an id outside that range sets the workspace status, reported as
+ * OPD_ERR_INVALID_ARG by opd_kl_get_status). Workspace as for opd_kl_forward. bf16 only
+ * (OPD_ERR_UNSUPPORTED otherwise). */
+opd_status opd_score_tokens(const opd_problem* problem, const void* H, const void* W, const int32_t* tokens,
+                            const uint8_t* mask, float* lse_out, float* logp_out, void* workspace,
+                            size_t workspace_bytes, void* stream);
+
+/* Constants of the dual-clip surrogate; NULL means the paper's values
+ * (delta = 0.2, kappa = 3, log-ratio clip 20; Appendix B.4). */
+typedef struct {
+  float delta;           /* clipping width of the ratio, 0 <= delta < 1 */
+  float kappa;           /* dual-clip constant, > 0 */
+  float log_ratio_clip;  /* bound on |log ratio| before exponentiation, > 0 */
+} opd_surrogate_params;
+
+/* The sampled-token surrogate the paper optimises (Appendix B.4, Eq. opd-token-advantage,
+ * opd-ratio, opd-dual-clip, opd-surrogate), forward and backward, student side:
+ *   logp_i = log pi_student(tokens[i])                       (full-vocabulary softmax of H_s W_s^T / tau)
+ *   A_i    = logp_teacher[i] - logp_old[i]                    (stop-gradient)
+ *   rho_i  = exp(clip(logp_i - logp_old[i], -c, c))
+ *   l_clip = -min(rho A, clip(rho, 1 - delta, 1 + delta) A);  l_i = min(l_clip, -kappa A) if A < 0
+ *   L = sum_i weights[i] l_i   (weights: e.g. opd_seq_mean_token_mean_weights)
+ * Writes loss_out[i] = l_i and logp_out[i] (zeros on rows with mask 0), dH_s [T, d_s] =
+ * dL/dH_s (zeros on masked rows) and dW_s [V, d_s] = dL/dW_s (added to dW_s when
+ * accumulate_dW != 0). The teacher enters only through logp_teacher (frozen). Sizes and
+ * workspace as for opd_kl_fwd_bwd with d_t unused; bf16 only. Token ids as for
+ * opd_score_tokens. */
+opd_status opd_surrogate_fwd_bwd(const opd_problem* problem, const void* H_s, const void* W_s,
+                                 const int32_t* tokens, const float* logp_old, const float* logp_teacher,
+                                 const uint8_t* mask, const float* weights, const opd_surrogate_params* params,
+                                 float* loss_out, float* logp_out, float* dH_s, float* dW_s, int accumulate_dW,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
 /* Largest T that opd_kl_forward_noalloc accepts. */
 #define OPD_KL_NOALLOC_MAX_ROWS 4096
 
@@ -137,8 +178,8 @@ opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t*
                                            float* w_out);
 
 /* Reads and clears the device status word in the workspace, after
- * synchronising the stream: OPD_OK, or OPD_ERR_TIMEOUT if a bounded wait in the
- * last call ran out. */
+ * synchronising the stream: OPD_OK, OPD_ERR_TIMEOUT if a bounded wait in the last
+ * call ran out, or OPD_ERR_INVALID_ARG if a token id was outside [0, V). */
 opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stream);
 
 /* Self-test of the bounded-wait machinery: launches one kernel that waits on a

@@ -241,12 +241,13 @@ opd_status check_inputs(const Call& c, const void* H_s, const void* H_t, const v
   return OPD_OK;
 }
 
-// Row compaction plus (bf16) the gather of supervised rows.
+// Row compaction plus (bf16) the gather of supervised rows (H_t may be null: one head).
 opd_status prologue(const Call& c, const void* H_s, const void* H_t, const uint8_t* mask) {
   OPD_CUDA(timed("compact", c.s, [&] { return launch_compact(mask, (int32_t)c.p.T, c.idx(), c.pos(), c.ctrl(), c.s); }));
   if (c.p.dtype == OPD_DTYPE_BF16) {
+    const int32_t d_t = H_t ? (int32_t)c.p.d_t : 0;
     OPD_CUDA(timed("gather", c.s, [&] {
-      return launch_gather_bf16(H_s, H_t, (int32_t)c.p.d_s, (int32_t)c.p.d_t, c.idx(), c.ctrl(), c.ws + c.L.hs_g,
+      return launch_gather_bf16(H_s, H_t, (int32_t)c.p.d_s, d_t, c.idx(), c.ctrl(), c.ws + c.L.hs_g,
                                 c.ws + c.L.ht_g, (int32_t)c.L.T_pad, c.dev.sm_count, c.s);
     }));
   }
@@ -320,6 +321,8 @@ opd_status forward_body(const Call& c, const Maps& m, float* kl_out, float* stat
   return OPD_OK;
 }
 
+opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s, int accumulate_dW);
+
 opd_status backward_body(const Call& c, const Maps& m, const float* stats, const float* grad_kl, float* dH_s,
                          float* dW_s, int accumulate_dW) {
   FusedParams fp = fused_params(c);
@@ -330,6 +333,12 @@ opd_status backward_body(const Call& c, const Maps& m, const float* stats, const
   OPD_CUDA(timed("fused_logits_bwd", c.s, [&] {
     return launch_fused_backward(m.hs, m.ht, m.ws, m.wt, m.dz_store, fp, c.dev.sm_count, c.s);
   }));
+  return gradient_gemms(c, m, dH_s, dW_s, accumulate_dW);
+}
+
+// dH_s = dZ W_s (split-K partial sums, then scattered back to the T rows) and
+// dW_s (+)= dZ^T H_s, from the bf16 dz the fused backward wrote.
+opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s, int accumulate_dW) {
   float* dhg = reinterpret_cast<float*>(c.ws + c.L.dh_g);
   OPD_CUDA(timed("zero_rows", c.s, [&] {
     return launch_zero_rows(dhg, (int32_t)c.p.d_s, c.ctrl(), (int32_t)c.L.T_pad, c.dev.sm_count, c.s);
@@ -407,9 +416,83 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
   return finish_call(c);
 }
 
+// Single-head path: compaction, gather of the head's rows, fused forward statistics,
+// then the per-token finish (and, for the surrogate, the student backward).
+opd_status head_call(const opd_problem* problem, const void* H, const void* W, const int32_t* tokens,
+                     const uint8_t* mask, float* lse_out, float* logp_out, const float* logp_old,
+                     const float* logp_teacher, const float* weights, const opd_surrogate_params* sp,
+                     float* loss_out, float* dH, float* dW, int accumulate_dW, void* workspace, size_t ws_bytes,
+                     void* stream, bool surrogate) {
+  Call c;
+  OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream));
+  if (c.p.dtype != OPD_DTYPE_BF16) return OPD_ERR_UNSUPPORTED;
+  const int64_t T = c.p.T;
+  if (!W || !aligned(W, 16) || !aligned(H, 16)) return OPD_ERR_INVALID_ARG;
+  if (T > 0 && (!H || !tokens || !mask || !logp_out)) return OPD_ERR_INVALID_ARG;
+  if (!surrogate && T > 0 && !lse_out) return OPD_ERR_INVALID_ARG;
+  if (surrogate) {
+    if (!dW || !aligned(dW, 16) || !aligned(dH, 16)) return OPD_ERR_INVALID_ARG;
+    if (T > 0 && (!logp_old || !logp_teacher || !weights || !loss_out || !dH)) return OPD_ERR_INVALID_ARG;
+    if (sp && (!(sp->delta >= 0.0f && sp->delta < 1.0f) || !(sp->kappa > 0.0f) || !(sp->log_ratio_clip > 0.0f)))
+      return OPD_ERR_INVALID_ARG;
+  }
+  OPD_TRY(prologue(c, H, nullptr, mask));
+  Maps m;
+  OPD_TRY(encode_maps(c, W, W, dW, m, surrogate));
+  FusedParams fp = fused_params(c);
+  OPD_CUDA(timed("head_logits_fwd", c.s, [&] { return launch_head_forward(m.hs, m.ws, fp, c.dev.sm_count, c.s); }));
+  HeadRowsParams hp{};
+  hp.ctrl = c.ctrl();
+  hp.ctrl_rw = c.ctrl();
+  hp.partials = fp.partials;
+  hp.T = (int32_t)T;
+  hp.T_pad = (int32_t)c.L.T_pad;
+  hp.V = (int32_t)c.p.V;
+  hp.d = (int32_t)c.p.d_s;
+  hp.pos = c.pos();
+  hp.H_g = reinterpret_cast<const __nv_bfloat16*>(c.ws + c.L.hs_g);
+  hp.W = static_cast<const __nv_bfloat16*>(W);
+  hp.tokens = tokens;
+  hp.inv_tau = 1.0f / c.p.temperature;
+  hp.lse_out = lse_out;
+  hp.logp_out = logp_out;
+  hp.surrogate = surrogate ? 1 : 0;
+  hp.logp_old = logp_old;
+  hp.logp_teacher = logp_teacher;
+  hp.weights = weights;
+  hp.delta = sp ? sp->delta : 0.2f;
+  hp.kappa = sp ? sp->kappa : 3.0f;
+  hp.clip = sp ? sp->log_ratio_clip : 20.0f;
+  hp.loss_out = loss_out;
+  hp.rowc = reinterpret_cast<float4*>(c.ws + c.L.rowc);
+  OPD_CUDA(timed("head_rows", c.s, [&] { return launch_head_rows(hp, c.dev.sm_count, c.s); }));
+  if (surrogate) {
+    OPD_CUDA(timed("head_logits_bwd", c.s,
+                   [&] { return launch_head_backward(m.hs, m.ws, m.dz_store, fp, c.dev.sm_count, c.s); }));
+    OPD_TRY(gradient_gemms(c, m, dH, dW, accumulate_dW));
+  }
+  return finish_call(c);
+}
+
 }  // namespace
 
 extern "C" {
+
+opd_status opd_score_tokens(const opd_problem* problem, const void* H, const void* W, const int32_t* tokens,
+                            const uint8_t* mask, float* lse_out, float* logp_out, void* workspace,
+                            size_t workspace_bytes, void* stream) {
+  return head_call(problem, H, W, tokens, mask, lse_out, logp_out, nullptr, nullptr, nullptr, nullptr, nullptr,
+                   nullptr, nullptr, 0, workspace, workspace_bytes, stream, false);
+}
+
+opd_status opd_surrogate_fwd_bwd(const opd_problem* problem, const void* H_s, const void* W_s,
+                                 const int32_t* tokens, const float* logp_old, const float* logp_teacher,
+                                 const uint8_t* mask, const float* weights, const opd_surrogate_params* params,
+                                 float* loss_out, float* logp_out, float* dH_s, float* dW_s, int accumulate_dW,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+  return head_call(problem, H_s, W_s, tokens, mask, nullptr, logp_out, logp_old, logp_teacher, weights, params,
+                   loss_out, dH_s, dW_s, accumulate_dW, workspace, workspace_bytes, stream, true);
+}
 
 size_t opd_kl_workspace_size(const opd_problem* problem) {
   if (!problem) return 0;
@@ -476,6 +559,7 @@ opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stre
   const uint32_t zero = 0;
   if (cudaMemcpy(&ctrl->status, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess) return OPD_ERR_CUDA;
   if (st & kDevTimeout) return OPD_ERR_TIMEOUT;
+  if (st & kDevBadToken) return OPD_ERR_INVALID_ARG;
   if (st & kDevBadShape) return OPD_ERR_UNSUPPORTED;
   return OPD_OK;
 }

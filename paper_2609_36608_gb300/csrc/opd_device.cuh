@@ -15,6 +15,7 @@ namespace opd {
 enum : uint32_t {
   kDevTimeout = 1u,    // a bounded wait ran out
   kDevBadShape = 2u,   // a kernel found a size it cannot handle
+  kDevBadToken = 4u,   // a token id outside [0, V)
 };
 
 // Control block at the head of the workspace.

@@ -41,7 +41,7 @@ constexpr int kNEpi = 8;   // epilogue warps
 constexpr int kColsPerWarp = kBN / 2;
 constexpr int kThreads = 64 + 32 * kNEpi;
 
-template <bool BWD, bool PAIR>
+template <bool BWD, bool PAIR, int HEADS>
 struct FusedCfg {
   static constexpr int kTileRows = PAIR ? 2 * kRowTile : kRowTile;  // rows per tile (whole pair)
   static constexpr int kBRows = PAIR ? kBN / 2 : kBN;              // W rows staged by one CTA
@@ -57,6 +57,7 @@ struct FusedCfg {
   static constexpr size_t kSmem = kFixed + (size_t)kStages * kStageBytes;
   static constexpr int kFreeCount = PAIR ? 2 * kNEpi : kNEpi;  // epilogue warps that release TMEM
   static_assert(kStages >= 3, "pipeline depth");
+  static_assert(HEADS == 1 || HEADS == 2, "one head (scoring, surrogate) or two (reverse KL)");
 };
 
 // Unit u -> (row tile, vocabulary tile range). Units are grouped by `G` row tiles
@@ -193,12 +194,65 @@ __device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kCol
                  w[4 * jj + 3]);
 }
 
-template <bool BWD, bool PAIR>
+// One head: 32 columns of one row folded into the running base-2 (max, sum).
+template <bool PARTIAL>
+__device__ __forceinline__ void fold_chunk1(const uint32_t (&rs)[32], int nvalid, float k2, float& m, float& S) {
+  float cm = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (!PARTIAL || j < nvalid) cm = fmaxf(cm, __uint_as_float(rs[j]));
+  const float nm = fmaxf(m, cm * k2);
+  S *= exp2f(m - nm);
+  m = nm;
+#pragma unroll
+  for (int j = 0; j < 32; ++j)
+    if (!PARTIAL || j < nvalid) S += exp2f(fmaf(__uint_as_float(rs[j]), k2, -m));
+}
+
+template <int C>
+__device__ __forceinline__ void fwd_chunk1(uint32_t ts, int nvalid_base, float k2, float& m, float& S) {
+  uint32_t rs[32];
+  tmem_ld32(ts + C * 32, rs);
+  const int nvalid = nvalid_base - C * 32;
+  if (nvalid >= 32)
+    fold_chunk1<false>(rs, 32, k2, m, S);
+  else if (nvalid > 0)
+    fold_chunk1<true>(rs, nvalid, k2, m, S);
+}
+
+// One head, backward of a loss on the sampled token's log-probability:
+// dz = coef (1[col = x] - p), p = 2^(z k2 - b1); bf16 into the warp's staging box.
+template <int C>
+__device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, float coef, int x_rel, uint32_t stg,
+                                           int lane) {
+  uint32_t rs[32];
+  tmem_ld32(ts + C * 32, rs);
+  uint32_t w[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    float dz2[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int col = C * 32 + 2 * j + e;
+      const float p = exp2f(fmaf(__uint_as_float(rs[2 * j + e]), k2, -b1));
+      dz2[e] = coef * ((col == x_rel ? 1.0f : 0.0f) - p);
+    }
+    w[j] = pack_bf16x2(dz2[0], dz2[1]);
+  }
+  const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
+  const uint32_t jb = (uint32_t)(C & 1) * 4u;
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj)
+    st_shared_v4(box + sw128_offset((uint32_t)lane, jb + jj), w[4 * jj], w[4 * jj + 1], w[4 * jj + 2],
+                 w[4 * jj + 3]);
+}
+
+template <bool BWD, bool PAIR, int HEADS>
 __global__ void __launch_bounds__(kThreads, 1)
     k_fused_logits(const __grid_constant__ CUtensorMap tm_hs, const __grid_constant__ CUtensorMap tm_ht,
                    const __grid_constant__ CUtensorMap tm_ws, const __grid_constant__ CUtensorMap tm_wt,
                    const __grid_constant__ CUtensorMap tm_dz, const FusedParams p) {
-  using C = FusedCfg<BWD, PAIR>;
+  using C = FusedCfg<BWD, PAIR, HEADS>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* stage_base = smem;
@@ -206,9 +260,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* merge = reinterpret_cast<float*>(staging + kNEpi * C::kStagingPerWarp);
   uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(merge) + C::kMergeBytes);
   uint64_t* empty = full + C::kStages;
-  uint64_t* acc_full = empty + C::kStages;  // both segments of a tile computed
-  uint64_t* t_free = acc_full + 1;          // teacher columns read by every epilogue warp
-  uint64_t* s_free = t_free + 1;            // student columns read by every epilogue warp
+  // acc_full[0]: both segments of a tile computed (two heads). One head: acc_full[slot]
+  // for TMEM slot 0 / 1 (columns 0-255 / 256-511, alternate tiles), so each barrier runs
+  // at most one phase ahead of the epilogue that waits on it.
+  uint64_t* acc_full = empty + C::kStages;
+  // Two heads: teacher / student columns read by every epilogue warp. One head: slot 0 /
+  // slot 1 read by every epilogue warp.
+  uint64_t* t_free = acc_full + 2;
+  uint64_t* s_free = t_free + 1;
   uint64_t* mma_done = s_free + 1;
   uint64_t* merge_full = mma_done + 1;      // [4]
   uint64_t* merge_empty = merge_full + 4;   // [4]
@@ -227,7 +286,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(acc_full, 1);
+    mbar_init(&acc_full[0], 1);
+    mbar_init(&acc_full[1], 1);
     mbar_init(t_free, C::kFreeCount);
     mbar_init(s_free, C::kFreeCount);
     mbar_init(mma_done, 1);
@@ -283,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row0 = rt * C::kTileRows + (int)rank * kRowTile;
         for (int vt = vb; ok && vt < ve; ++vt) {
           const int wrow0 = vt * kBN + (int)rank * C::kBRows;
-          for (int seg = 0; ok && seg < 2; ++seg) {  // teacher, then student
+          for (int seg = 2 - HEADS; ok && seg < 2; ++seg) {  // teacher (two heads), then student
             const CUtensorMap* ta = seg ? &tm_hs : &tm_ht;
             const CUtensorMap* tb = seg ? &tm_ws : &tm_wt;
             const int nk = seg ? nks : nkt;
@@ -332,14 +392,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
         for (int vt = vb; ok && vt < ve; ++vt, ++lt) {
-          const uint32_t free_par = ((uint32_t)lt & 1u) ^ 1u;  // previous tile's release
-          for (int seg = 0; ok && seg < 2; ++seg) {
-            if (!mbar_wait(seg ? s_free : t_free, free_par, status, lim)) {
+          for (int seg = 2 - HEADS; ok && seg < 2; ++seg) {
+            // two heads: each segment reuses its columns every tile; one head: the
+            // tile alternates between two column slots
+            const int slot = HEADS == 2 ? seg : (lt & 1);
+            const uint32_t free_par = HEADS == 2 ? (((uint32_t)lt & 1u) ^ 1u) : ((((uint32_t)lt >> 1) & 1u) ^ 1u);
+            if (!mbar_wait(slot ? s_free : t_free, free_par, status, lim)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t d_tmem = seg ? tmem_s : tmem_t;
+            const uint32_t d_tmem = slot ? tmem_s : tmem_t;
             const int nk = seg ? nks : nkt;
             for (int kb = 0; kb < nk; ++kb) {
               if (!mbar_wait(&full[stage], phase, status, lim)) {
@@ -369,10 +432,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           if (ok) {
+            uint64_t* af = HEADS == 2 ? &acc_full[0] : &acc_full[lt & 1];
             if (PAIR)
-              umma_commit_pair_mc(acc_full, 0x3);
+              umma_commit_pair_mc(af, 0x3);
             else
-              umma_commit(acc_full);
+              umma_commit(af);
           }
         }
       }
@@ -403,21 +467,74 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row_base = rt * C::kTileRows + (int)rank * kRowTile;
       const int row = row_base + row_in_tile;
       float ms = -INFINITY, Ss = 0.f, A = 0.f, mt = -INFINITY, St = 0.f;
-      // backward row constants: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc)
+      // backward row constants. Two heads: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc).
+      // One head: dz = coef (1[col = x] - p_s) with coef = rowc.y and token x = rowc.z (bits).
       float b1 = 0.f, kc = 0.f, cc = 0.f;
+      int x_tok = -1;
       if (BWD) {
         const float4 rc = p.rowc[row];
         b1 = rc.x;
-        kc = rc.z * p.inv_tau;
-        cc = rc.z * rc.y;
+        if (HEADS == 2) {
+          kc = rc.z * p.inv_tau;
+          cc = rc.z * rc.y;
+        } else {
+          kc = rc.y;
+          x_tok = __float_as_int(rc.z);
+        }
       }
       for (int vt = vb; vt < ve; ++vt, ++lt) {
         // warp-uniform outcome: the TMEM loads below are .sync.aligned
-        if (!__all_sync(0xffffffffu, mbar_wait(acc_full, (uint32_t)lt & 1u, status, lim))) {
+        uint64_t* af = HEADS == 2 ? &acc_full[0] : &acc_full[lt & 1];
+        const uint32_t af_par = HEADS == 2 ? ((uint32_t)lt & 1u) : (((uint32_t)lt >> 1) & 1u);
+        if (!__all_sync(0xffffffffu, mbar_wait(af, af_par, status, lim))) {
           ok = false;
           break;
         }
         tc_fence_after();
+        if (HEADS == 1) {
+          const int slot = lt & 1;
+          const int col0 = vt * kBN + cbase;
+          const uint32_t ts = (slot ? tmem_s : tmem_t) + t_lane + (uint32_t)cbase;
+          if (!BWD) {
+            const int nv = p.V - col0;
+            fwd_chunk1<0>(ts, nv, p.k2, ms, Ss);
+            fwd_chunk1<1>(ts, nv, p.k2, ms, Ss);
+            fwd_chunk1<2>(ts, nv, p.k2, ms, Ss);
+            fwd_chunk1<3>(ts, nv, p.k2, ms, Ss);
+          } else {
+            const int x_rel = x_tok - col0;  // the token's column within this warp's 128
+            if (lane == 0) bulk_wait_read<1>();
+            __syncwarp();
+            bwd_chunk1<0>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            bwd_chunk1<1>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, row_base + q * 32);
+              bulk_commit();
+              bulk_wait_read<1>();
+            }
+            __syncwarp();
+            bwd_chunk1<2>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            bwd_chunk1<3>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, row_base + q * 32);
+              bulk_commit();
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            uint64_t* fb = slot ? s_free : t_free;
+            if (PAIR)
+              mbar_arrive_cluster(slot ? s_free_addr : t_free_addr);
+            else
+              mbar_arrive(fb);
+          }
+          continue;
+        }
         // teacher columns to registers, then release them to the next tile's MMAs
         uint32_t tv[kColsPerWarp];
         tmem_ld128(tmem_t + t_lane + (uint32_t)cbase, tv);
@@ -498,20 +615,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float mt1 = mb[3 * 32 + lane], St1 = mb[4 * 32 + lane];
         __syncwarp();
         if (lane == 0) mbar_arrive(&merge_empty[q]);
-        const float Ms = fmaxf(ms, ms1), Mt = fmaxf(mt, mt1);
+        const float Ms = fmaxf(ms, ms1);
         const float f0 = exp2f(ms - Ms), f1 = exp2f(ms1 - Ms);
         Ss = Ss * f0 + Ss1 * f1;
-        A = A * f0 + A1 * f1;
-        St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
         ms = Ms;
-        mt = Mt;
         const size_t plane = (size_t)p.T_pad;
         float* base = p.partials + (size_t)split * 5 * plane + row;
         base[0 * plane] = ms;
         base[1 * plane] = Ss;
-        base[2 * plane] = A;
-        base[3 * plane] = mt;
-        base[4 * plane] = St;
+        if (HEADS == 2) {
+          const float Mt = fmaxf(mt, mt1);
+          A = A * f0 + A1 * f1;
+          St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
+          mt = Mt;
+          base[2 * plane] = A;
+          base[3 * plane] = mt;
+          base[4 * plane] = St;
+        }
       }
     }
     if (BWD && lane == 0) bulk_wait_all<0>();
@@ -531,13 +651,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <bool BWD, bool PAIR>
+template <bool BWD, bool PAIR, int HEADS>
 cudaError_t launch_fused_impl(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                               const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
                               cudaStream_t s) {
-  using C = FusedCfg<BWD, PAIR>;
+  using C = FusedCfg<BWD, PAIR, HEADS>;
   static_assert(C::kSmem <= 232448, "shared memory budget");
-  auto kern = k_fused_logits<BWD, PAIR>;
+  auto kern = k_fused_logits<BWD, PAIR, HEADS>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::kSmem);
   if (e != cudaSuccess) return e;
   if (!PAIR) {
@@ -568,13 +688,13 @@ cudaError_t launch_fused_impl(const CUtensorMap& hs, const CUtensorMap& ht, cons
   return cudaGetLastError();
 }
 
-template <bool BWD>
+template <bool BWD, int HEADS>
 cudaError_t launch_fused_mode(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                               const CUtensorMap& wt, const CUtensorMap& dz, const FusedParams& p, int grid,
                               cudaStream_t s) {
   switch (fused_mode(p)) {
-    case kFusedBN256: return launch_fused_impl<BWD, false>(hs, ht, ws, wt, dz, p, grid, s);
-    case kFusedPair256: return launch_fused_impl<BWD, true>(hs, ht, ws, wt, dz, p, grid, s);
+    case kFusedBN256: return launch_fused_impl<BWD, false, HEADS>(hs, ht, ws, wt, dz, p, grid, s);
+    case kFusedPair256: return launch_fused_impl<BWD, true, HEADS>(hs, ht, ws, wt, dz, p, grid, s);
   }
   return cudaErrorInvalidValue;
 }
@@ -583,13 +703,23 @@ cudaError_t launch_fused_mode(const CUtensorMap& hs, const CUtensorMap& ht, cons
 
 cudaError_t launch_fused_forward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                  const CUtensorMap& wt, const FusedParams& p, int grid, cudaStream_t s) {
-  return launch_fused_mode<false>(hs, ht, ws, wt, hs, p, grid, s);
+  return launch_fused_mode<false, 2>(hs, ht, ws, wt, hs, p, grid, s);
 }
 
 cudaError_t launch_fused_backward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                   const CUtensorMap& wt, const CUtensorMap& dz_store, const FusedParams& p,
                                   int grid, cudaStream_t s) {
-  return launch_fused_mode<true>(hs, ht, ws, wt, dz_store, p, grid, s);
+  return launch_fused_mode<true, 2>(hs, ht, ws, wt, dz_store, p, grid, s);
+}
+
+cudaError_t launch_head_forward(const CUtensorMap& h, const CUtensorMap& w, const FusedParams& p, int grid,
+                                cudaStream_t s) {
+  return launch_fused_mode<false, 1>(h, h, w, w, h, p, grid, s);
+}
+
+cudaError_t launch_head_backward(const CUtensorMap& h, const CUtensorMap& w, const CUtensorMap& dz_store,
+                                 const FusedParams& p, int grid, cudaStream_t s) {
+  return launch_fused_mode<true, 1>(h, h, w, w, dz_store, p, grid, s);
 }
 
 }  // namespace opd

@@ -3,6 +3,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -51,6 +52,28 @@ struct GemmParams {
   uint64_t wait_limit_ns;
 };
 
+// Per-token finish of single-head scoring and of the sampled-token surrogate (opd_surrogate.cu).
+struct HeadRowsParams {
+  const Ctrl* ctrl;             // R and the forward's split count
+  Ctrl* ctrl_rw;                // status word (bad token ids)
+  const float* partials;        // [split][5][T_pad] base-2 statistics (planes 0, 1 used)
+  int32_t T, T_pad, V, d;
+  const int32_t* pos;           // token row -> gathered rank or -1
+  const __nv_bfloat16* H_g;     // gathered rows [T_pad, d]
+  const __nv_bfloat16* W;       // head [V, d]
+  const int32_t* tokens;        // [T]
+  float inv_tau;
+  float* lse_out;               // [T] (may be null)
+  float* logp_out;              // [T] (may be null)
+  int32_t surrogate;            // 1: also the dual-clip loss and the backward constants
+  const float* logp_old;        // [T]
+  const float* logp_teacher;    // [T]
+  const float* weights;         // [T] upstream weight of each token's loss
+  float delta, kappa, clip;
+  float* loss_out;              // [T]
+  float4* rowc;                 // [T_pad] (lse log2 e, coef, token bits, 0)
+};
+
 // aux kernels (opd_aux.cu)
 cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t* pos, Ctrl* ctrl,
                            cudaStream_t s);
@@ -81,6 +104,14 @@ cudaError_t launch_fused_forward(const CUtensorMap& hs, const CUtensorMap& ht, c
 cudaError_t launch_fused_backward(const CUtensorMap& hs, const CUtensorMap& ht, const CUtensorMap& ws,
                                   const CUtensorMap& wt, const CUtensorMap& dz_store, const FusedParams& p,
                                   int grid, cudaStream_t s);
+// Single-head variants (scoring, surrogate): the head's rows and weights come in the
+// student slots; forward writes base-2 (max, sum) partials, backward writes
+// dz = coef (1[k = x] - p) from rowc = (lse log2 e, coef, token bits, 0).
+cudaError_t launch_head_forward(const CUtensorMap& h, const CUtensorMap& w, const FusedParams& p, int grid,
+                                cudaStream_t s);
+cudaError_t launch_head_backward(const CUtensorMap& h, const CUtensorMap& w, const CUtensorMap& dz_store,
+                                 const FusedParams& p, int grid, cudaStream_t s);
+cudaError_t launch_head_rows(const HeadRowsParams& p, int n_sm, cudaStream_t s);
 // C = A * B^T with A [M, K] and B [N, K] given through tensor maps; a_mn / b_mn select
 // MN-major operand tiles (the operand's contiguous dimension is M or N, not K).
 cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,

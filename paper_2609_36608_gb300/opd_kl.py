@@ -39,6 +39,10 @@ class opd_kernel_time(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int64), ("total_ms", ctypes.c_double)]
 
 
+class opd_surrogate_params(ctypes.Structure):
+    _fields_ = [("delta", ctypes.c_float), ("kappa", ctypes.c_float), ("log_ratio_clip", ctypes.c_float)]
+
+
 class OpdError(RuntimeError):
     def __init__(self, status: int, what: str):
         super().__init__(f"{what}: {opd_status_string(status)} ({status})")
@@ -62,6 +66,9 @@ def _load() -> ctypes.CDLL:
         "opd_kl_get_status": (i32, [vp, sz, vp]),
         "opd_kl_selftest_timeout": (i32, [vp, sz, ctypes.c_uint64, vp]),
         "opd_status_string": (ctypes.c_char_p, [i32]),
+        "opd_score_tokens": (i32, [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
+        "opd_surrogate_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, vp, ctypes.POINTER(opd_surrogate_params),
+                                        vp, vp, vp, vp, i32, vp, sz, vp]),
         "opd_kl_profile_start": (i32, []),
         "opd_kl_profile_stop": (i32, [ctypes.POINTER(opd_kernel_time), i32, ctypes.POINTER(i32)]),
     }
@@ -149,6 +156,24 @@ def opd_kl_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, grad_kl, kl_out, stats, dH
                                _ptr(grad_kl), _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s),
                                int(bool(accumulate_dW)), _ptr(workspace), workspace.numel(), _stream(stream)),
            "opd_kl_fwd_bwd")
+
+
+def opd_score_tokens(problem, H, W, tokens, mask, lse_out, logp_out, workspace, stream=None) -> None:
+    """Log-partition and log-probability of the given tokens under one head (d = problem.d_s)."""
+    _check(_lib.opd_score_tokens(ctypes.byref(problem), _ptr(H), _ptr(W), _ptr(tokens), _ptr(mask), _ptr(lse_out),
+                                 _ptr(logp_out), _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_score_tokens")
+
+
+def opd_surrogate_fwd_bwd(problem, H_s, W_s, tokens, logp_old, logp_teacher, mask, weights, loss_out, logp_out,
+                          dH_s, dW_s, accumulate_dW: bool, workspace, params=None, stream=None) -> None:
+    """Sampled-token dual-clip surrogate, forward and backward (student side)."""
+    pp = ctypes.byref(params) if params is not None else None
+    _check(_lib.opd_surrogate_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(W_s), _ptr(tokens), _ptr(logp_old),
+                                      _ptr(logp_teacher), _ptr(mask), _ptr(weights), pp, _ptr(loss_out),
+                                      _ptr(logp_out), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
+                                      _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_surrogate_fwd_bwd")
 
 
 def opd_seq_mean_token_mean_weights(seg_id, mask, eps: float = 1e-8) -> np.ndarray:

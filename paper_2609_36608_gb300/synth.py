@@ -34,6 +34,7 @@ STREAM_H_S, STREAM_H_T, STREAM_W_S, STREAM_W_T = 1, 2, 3, 4
 STREAM_H_T_EXTRA, STREAM_W_T_EXTRA = 5, 6
 STREAM_LAYOUT = 7
 STREAM_G = 8
+STREAM_TOKENS = 9
 
 
 def pcg_hash_int(x: int) -> int:
@@ -340,6 +341,12 @@ def uniform_weights(seed: int, T: int) -> np.ndarray:
     """Seeded upstream weights in [0.5, 1.5) for parity tests (float64)."""
     bits = uniform_bits(stream_key(seed, STREAM_G), 0, T, "cpu")
     return 0.5 + (bits.to(torch.float64) + 0.5).numpy() * (2.0 ** -32)
+
+
+def token_ids(seed: int, T: int, V: int) -> np.ndarray:
+    """Seeded sampled-token ids in [0, V) (int32)."""
+    bits = uniform_bits(stream_key(seed, STREAM_TOKENS), 0, T, "cpu").numpy()
+    return ((bits.astype(np.uint64) * np.uint64(V)) >> np.uint64(32)).astype(np.int32)
 
 
 def bf16_bits(t: torch.Tensor) -> np.ndarray:

@@ -1,0 +1,206 @@
+"""GPU parity of token scoring and the sampled-token surrogate (Appendix B.4) against
+the float64 oracle, through the C ABI.
+
+Tolerances: log-partition and log-probability |gpu - oracle| <= 1e-4 + 1e-4 |oracle|;
+per-token surrogate loss |gpu - oracle| <= 1e-4 + 2e-3 |oracle|; dH_s and dW_s within
+1e-2 relative Frobenius error (bf16 inputs, fp32 accumulation, bf16 dz).
+
+The surrogate's gradient is piecewise (ratio clip, dual clip, log-ratio clip), so a
+branch decision taken in fp32 on the GPU and in fp64 in the oracle could differ for a
+token sitting on a kink. The small cases therefore build the behaviour-policy
+log-probabilities from the oracle's own scores, keeping every token's log-ratio at least
+0.02 away from ln 0.8, ln 1.2 and ln 3 (the GPU's log-probabilities differ from the
+oracle's by ~1e-5).
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36608_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+EDGES = np.log([0.8, 1.2, 3.0])
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+    return opd_kl
+
+
+@pytest.fixture(params=["bn256", "pair256"])
+def tiling(request, monkeypatch):
+    monkeypatch.setenv("OPD_KL_FUSED", request.param)
+    return request.param
+
+
+def _case(**kw):
+    base = dict(name="head", T=700, d_s=256, d_t=384, V=1000, tau=0.7, n_traj=7, traj_len=100, seed=31)
+    base.update(kw)
+    return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
+
+
+def _rel(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _close(got, want, abs_tol, rel_tol, what):
+    excess = np.abs(np.asarray(got, np.float64) - want) - (abs_tol + rel_tol * np.abs(want))
+    assert excess.max() <= 0, f"{what}: worst excess {excess.max():.3e} at {int(excess.argmax())}"
+
+
+def _score(lib, w, H, W, tokens, mask):
+    prob = lib.make_problem(w.T, H.shape[1], H.shape[1], w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    lse = torch.full((w.T,), float("nan"), device="cuda")
+    lp = torch.full((w.T,), float("nan"), device="cuda")
+    lib.opd_score_tokens(prob, H, W, torch.from_numpy(tokens).cuda(), torch.from_numpy(mask).cuda(), lse, lp, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    return lse.cpu().numpy(), lp.cpu().numpy()
+
+
+def _surrogate(lib, w, x, tokens, logp_old, logp_teacher, mask, weights, accumulate=False, dW_init=None):
+    prob = lib.make_problem(w.T, w.d_s, w.d_s, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    f32 = lambda a: torch.from_numpy(np.asarray(a, np.float32)).cuda()
+    loss = torch.full((w.T,), float("nan"), device="cuda")
+    lp = torch.full((w.T,), float("nan"), device="cuda")
+    dH = torch.full((w.T, w.d_s), float("nan"), device="cuda")
+    dW = torch.full((w.V, w.d_s), float("nan"), device="cuda") if dW_init is None else dW_init.clone()
+    lib.opd_surrogate_fwd_bwd(prob, x["H_s"], x["W_s"], torch.from_numpy(tokens).cuda(), f32(logp_old),
+                              f32(logp_teacher), torch.from_numpy(mask).cuda(), f32(weights), loss, lp, dH, dW,
+                              accumulate, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    return loss.cpu().numpy(), lp.cpu().numpy(), dH.cpu().numpy(), dW.cpu().numpy()
+
+
+def _clear_offsets(seed, n):
+    rng = np.random.default_rng(seed)
+    out = np.empty(n)
+    for i in range(n):
+        while True:
+            r = rng.uniform(-0.6, 1.4)
+            if np.min(np.abs(r - EDGES)) > 0.02:
+                out[i] = r
+                break
+    return out
+
+
+def test_score_tokens_small(lib, oracle_mod, tiling):
+    w = _case()
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    for H, W in ((x["H_s"], x["W_s"]), (x["H_t"], x["W_t"])):
+        lse, lp = _score(lib, w, H, W, tokens, lay.mask)
+        sup = lay.mask != 0
+        ref_lse, ref_lp = oracle_mod.score(synth.host_values(H), synth.host_values(W), tokens, w.tau,
+                                           rows=np.flatnonzero(sup))
+        _close(lse[sup], ref_lse, 1e-4, 1e-4, "lse")
+        _close(lp[sup], ref_lp, 1e-4, 1e-4, "logp")
+        assert (lse[~sup] == 0).all() and (lp[~sup] == 0).all()
+
+
+def test_surrogate_small(lib, oracle_mod, tiling):
+    w = _case(T=600, d_s=192, V=1237, tau=0.9, n_traj=6, seed=32)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    _, lp_ref = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = (lp_ref - _clear_offsets(1, w.T)).astype(np.float32)
+    adv = np.random.default_rng(2).choice([-1.0, 1.0], w.T) * np.random.default_rng(3).uniform(0.2, 1.5, w.T)
+    logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
+    weights = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask).astype(np.float32)
+    loss, lp, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, lay.mask, weights)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               lay.mask, weights.astype(np.float64), w.tau)
+    sup = lay.mask != 0
+    _close(lp[sup], ref.logp_s[sup], 1e-4, 1e-4, "logp")
+    _close(loss, ref.loss, 1e-4, 2e-3, "loss")
+    assert (loss[~sup] == 0).all() and (dH[~sup] == 0).all()
+    assert _rel(dH, ref.dH_s) <= 1e-2, _rel(dH, ref.dH_s)
+    assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
+
+
+def test_surrogate_on_policy_and_accumulate(lib, oracle_mod):
+    # rho = 1: the surrogate's gradient is the policy gradient -A (1[k = x] - p) / tau
+    w = _case(T=300, d_s=128, V=2048, tau=1.0, n_traj=3, seed=33)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    _, lp_ref = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = lp_ref.astype(np.float32)
+    logp_teacher = (lp_ref + 0.5).astype(np.float32)
+    weights = np.ones(w.T, np.float32)
+    init = torch.randn(w.V, w.d_s, device="cuda", generator=torch.Generator("cuda").manual_seed(1))
+    loss, lp, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, lay.mask, weights, True, init)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               lay.mask, weights.astype(np.float64), w.tau)
+    sup = lay.mask != 0
+    _close(loss[sup], -0.5 * np.ones(sup.sum()), 1e-3, 0, "on-policy loss")
+    assert _rel(dW - init.cpu().numpy(), ref.dW_s) <= 1e-2
+    assert _rel(dH, ref.dH_s) <= 1e-2
+
+
+def test_out_of_range_token_is_reported_not_read(lib):
+    w = _case(T=256, d_s=64, V=500, n_traj=2, traj_len=128, seed=34)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    tokens[np.flatnonzero(lay.mask)[3]] = w.V + 7
+    prob = lib.make_problem(w.T, w.d_s, w.d_s, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    lse = torch.empty(w.T, device="cuda")
+    lp = torch.empty(w.T, device="cuda")
+    lib.opd_score_tokens(prob, x["H_s"], x["W_s"], torch.from_numpy(tokens).cuda(),
+                         torch.from_numpy(lay.mask).cuda(), lse, lp, ws)
+    assert lib.opd_kl_get_status(ws) == lib.OPD_ERR_INVALID_ARG
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+
+
+@pytest.mark.parametrize("name", ["qwen3_1p7b"])
+def test_full_size_surrogate_and_scoring_sampled_rows(lib, oracle_mod, name):
+    w = synth.WORKLOADS[name]
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    sup = np.flatnonzero(lay.mask)
+    pick = np.unique(np.concatenate([sup[np.linspace(0, len(sup) - 1, 12).astype(int)], sup[:1], sup[-1:]]))
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    Ht, Wt = synth.host_values(x["H_t"]), synth.host_values(x["W_t"])
+    # teacher scoring at full size
+    lse_t, lp_t = _score(lib, w, x["H_t"], x["W_t"], tokens, lay.mask)
+    ref_lse, ref_lp = oracle_mod.score(Ht, Wt, tokens, w.tau, rows=pick)
+    _close(lse_t[pick], ref_lse, 1e-4, 1e-4, "teacher lse")
+    _close(lp_t[pick], ref_lp, 1e-4, 1e-4, "teacher logp")
+    # surrogate: synthetic teacher and behaviour log-probabilities, independent of the student
+    # (wide ratio spread; a fp32 / fp64 branch flip needs a token within ~1e-5 of a kink)
+    rng = np.random.default_rng(5)
+    logp_teacher = rng.normal(-7.0, 1.0, w.T).astype(np.float32)
+    logp_old = (logp_teacher.astype(np.float64) + rng.normal(0.0, 1.0, w.T)).astype(np.float32)
+    weights = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask).astype(np.float32)
+    loss, lp, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, lay.mask, weights)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               lay.mask, weights.astype(np.float64), w.tau, rows=pick, want_dW=False)
+    _close(lp[pick], ref.logp_s, 1e-4, 1e-4, "student logp")
+    _close(loss[pick], ref.loss, 1e-4, 2e-3, "loss")
+    assert _rel(dH[pick], ref.dH_s) <= 1e-2, _rel(dH[pick], ref.dH_s)
+    # dW_s with only a few supervised rows at full shape
+    mask2 = np.zeros_like(lay.mask)
+    mask2[pick[::2]] = 1
+    _, _, _, dW2 = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, mask2, weights)
+    ref2 = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                                mask2, weights.astype(np.float64), w.tau, rows=pick[::2], want_dH=False)
+    assert _rel(dW2, ref2.dW_s) <= 1e-2, _rel(dW2, ref2.dW_s)
