@@ -231,19 +231,33 @@ def run_reference(args):
     rows_per_step = args.ref_rows
     import oracle
     oracle.build()
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+
+    def one(rows):
+        if args.path == "kl":
+            oracle_rate(w, host, lay, g, rows, threads)
+        elif args.path == "score":
+            oracle.score(host["H_t"], host["W_t"], tokens, w.tau, rows=rows, n_threads=threads)
+        else:
+            oracle.surrogate(host["H_s"], host["W_s"], tokens, np.full(w.T, -7.0), np.full(w.T, -7.0), lay.mask,
+                             np.ones(w.T), w.tau, rows=rows, n_threads=threads)
+
     for i in range(args.warmup):
-        oracle_rate(w, host, lay, g, sample_rows(lay.mask, rows_per_step, 7 * i), threads)
+        one(sample_rows(lay.mask, rows_per_step, 7 * i))
     t0 = time.perf_counter()
     n = 0
     for i in range(args.steps):
         rows = sample_rows(lay.mask, rows_per_step, 13 * i + 1)
-        oracle_rate(w, host, lay, g, rows, threads)
+        one(rows)
         n += len(rows)
     dt = time.perf_counter() - t0
     value = n / dt
+    what = {"kl": "logits, KL, dH_s rows and their dW_s contribution",
+            "score": "teacher log-partition and token log-probabilities",
+            "surrogate": "student logits, dual-clip loss, dH_s rows and their dW_s contribution"}[args.path]
     sample = (f"{rows_per_step} supervised rows of {w.name} per step (full V={w.V}, d_s={w.d_s}, d_t={w.d_t}): "
-              f"logits, KL, dH_s rows and their dW_s contribution in float64")
-    out = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+              f"{what} in float64")
+    out = {"impl": "reference", "metric": PATH_METRICS[args.path], "value": value, "unit": UNIT, "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * dt / max(args.steps, 1),
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
            "data": "synthetic", "config": {"workload": w.name, "T": w.T, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
@@ -255,6 +269,105 @@ def run_reference(args):
 
 
 # ------------------------------------------------------------------ GPU arm
+
+PATH_METRICS = {
+    "kl": METRIC,
+    "surrogate": "response tokens/s, sampled-token dual-clip surrogate fwd+bwd (1 GB300)",
+    "score": "response tokens/s, teacher token scoring fwd (1 GB300)",
+}
+
+
+def path_setup(path, w, lay, x, dev, opd_kl):
+    """Per-step device inputs (the tensors the e2e leg copies from the host each step), the
+    step function over them, the output read back each step, and the step's FLOPs."""
+    R = int(lay.mask.sum())
+    mask = torch.from_numpy(lay.mask).to(dev)
+    weights = torch.from_numpy(opd_kl.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)).to(dev)
+    dtype = opd_kl.OPD_DTYPE_BF16 if w.dtype == "bf16" else opd_kl.OPD_DTYPE_F32
+    if path == "kl":
+        prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
+        ws = opd_kl.allocate_workspace(prob, dev)
+        kl, stats = torch.empty(w.T, device=dev), torch.empty(w.T, 3, device=dev)
+        dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+        inputs = {"H_s": x["H_s"], "H_t": x["H_t"], "mask": mask, "grad": weights}
+
+        def step(i):
+            opd_kl.opd_kl_fwd_bwd(prob, i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["grad"], kl, stats, dH,
+                                  dW, False, ws)
+        executed, algorithmic = step_flops(w, R)
+        return inputs, step, kl, ws, executed, algorithmic
+    tokens = torch.from_numpy(synth.token_ids(w.seed, w.T, w.V)).to(dev)
+    if path == "score":
+        prob = opd_kl.make_problem(w.T, w.d_t, w.d_t, w.V, dtype, w.tau)
+        ws = opd_kl.allocate_workspace(prob, dev)
+        lse, logp = torch.empty(w.T, device=dev), torch.empty(w.T, device=dev)
+        inputs = {"H_t": x["H_t"], "tokens": tokens, "mask": mask}
+
+        def step(i):
+            opd_kl.opd_score_tokens(prob, i["H_t"], x["W_t"], i["tokens"], i["mask"], lse, logp, ws)
+        fl = 2.0 * R * w.V * w.d_t
+        return inputs, step, logp, ws, fl, fl
+    # surrogate: synthetic teacher and behaviour log-probabilities (the teacher enters only there)
+    g = torch.Generator(device="cpu").manual_seed(w.seed)
+    logp_teacher = (torch.randn(w.T, generator=g) - 7.0).to(dev)
+    logp_old = (logp_teacher.cpu() + 0.3 * torch.randn(w.T, generator=g)).to(dev)
+    prob = opd_kl.make_problem(w.T, w.d_s, w.d_s, w.V, dtype, w.tau)
+    ws = opd_kl.allocate_workspace(prob, dev)
+    loss, logp = torch.empty(w.T, device=dev), torch.empty(w.T, device=dev)
+    dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+    inputs = {"H_s": x["H_s"], "tokens": tokens, "logp_old": logp_old, "logp_teacher": logp_teacher, "mask": mask,
+              "weights": weights}
+
+    def step(i):
+        opd_kl.opd_surrogate_fwd_bwd(prob, i["H_s"], x["W_s"], i["tokens"], i["logp_old"], i["logp_teacher"],
+                                     i["mask"], i["weights"], loss, logp, dH, dW, False, ws)
+    return inputs, step, loss, ws, 8.0 * R * w.V * w.d_s, 6.0 * R * w.V * w.d_s
+
+
+def path_kernel_flops(path, name, w, R):
+    if path == "kl":
+        return kernel_flops(name, w, R)
+    d = w.d_t if path == "score" else w.d_s
+    if name in ("head_logits_fwd", "head_logits_bwd"):
+        return 2.0 * R * w.V * d
+    if name in ("gemm_dH", "gemm_dW"):
+        return 2.0 * R * w.V * w.d_s
+    return None
+
+
+def path_cpu_baseline(path, w, lay, x, args):
+    """The oracle, as it stands, on a bounded row sample of the same workload."""
+    import oracle
+    oracle.build()
+    threads = os.cpu_count() or 1
+    rows = sample_rows(lay.mask, args.cpu_rows, 3)
+    if path == "kl":
+        host = host_inputs(x)
+        g = np.where(lay.mask != 0, opd_seq_weights(lay), 0.0)
+        rate, dt = oracle_rate(w, host, lay, g, rows, threads)
+        what = "float64 logits, KL, dH_s rows and their dW_s contribution"
+    else:
+        tokens = synth.token_ids(w.seed, w.T, w.V)
+        t0 = time.perf_counter()
+        if path == "score":
+            oracle.score(synth.host_values(x["H_t"]), synth.host_values(x["W_t"]), tokens, w.tau, rows=rows,
+                         n_threads=threads)
+            what = "float64 teacher log-partition and token log-probabilities"
+        else:
+            T = w.T
+            oracle.surrogate(synth.host_values(x["H_s"]), synth.host_values(x["W_s"]), tokens, np.full(T, -7.0),
+                             np.full(T, -7.0), lay.mask, np.ones(T), w.tau, rows=rows, n_threads=threads)
+            what = "float64 student logits, dual-clip loss, dH_s rows and their dW_s contribution"
+        dt = time.perf_counter() - t0
+        rate = len(rows) / dt
+    return {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{len(rows)} supervised rows of {w.name}: {what} ({dt:.1f} s)"}
+
+
+def opd_seq_weights(lay):
+    import oracle
+    return oracle.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+
 
 def run_gpu(args):
     world, rank, local = dist_env()
@@ -271,25 +384,13 @@ def run_gpu(args):
     lay = synth.layout(w)
     R = int(lay.mask.sum())
     x = synth.hidden_and_heads(w, dev)
-    grad_h = opd_kl.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)
-    mask = torch.from_numpy(lay.mask).to(dev)
-    grad = torch.from_numpy(grad_h).to(dev)
-    dtype = opd_kl.OPD_DTYPE_BF16 if w.dtype == "bf16" else opd_kl.OPD_DTYPE_F32
-    prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
-    ws = opd_kl.allocate_workspace(prob, dev)
-    kl = torch.empty(w.T, device=dev)
-    stats = torch.empty(w.T, 3, device=dev)
-    dH = torch.empty(w.T, w.d_s, device=dev)
-    dW = torch.empty(w.V, w.d_s, device=dev)
-
-    def step(H_s, H_t, m, gr):
-        opd_kl.opd_kl_fwd_bwd(prob, H_s, H_t, x["W_s"], x["W_t"], m, gr, kl, stats, dH, dW, False, ws)
+    inputs, step, result, ws, executed, algorithmic = path_setup(args.path, w, lay, x, dev, opd_kl)
 
     sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
         sampler.start()
     for _ in range(args.warmup):
-        step(x["H_s"], x["H_t"], mask, grad)
+        step(inputs)
     torch.cuda.synchronize()
     if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
         raise RuntimeError("device status after warm-up is not OK")
@@ -301,7 +402,7 @@ def run_gpu(args):
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record()
     for _ in range(args.steps):
-        step(x["H_s"], x["H_t"], mask, grad)
+        step(inputs)
     ev1.record()
     torch.cuda.synchronize()
     barrier(world)
@@ -314,27 +415,21 @@ def run_gpu(args):
     ms_step = ms / args.steps
     value = R * args.steps * world / (ms / 1000.0)
 
-    # end to end through the same C ABI: inputs from pinned host memory, KL back every step
-    H_s_h = x["H_s"].cpu().pin_memory()
-    H_t_h = x["H_t"].cpu().pin_memory()
-    mask_h = torch.from_numpy(lay.mask).pin_memory()
-    grad_hp = torch.from_numpy(grad_h).pin_memory()
-    kl_h = torch.empty(w.T, dtype=torch.float32).pin_memory()
-    H_s_d, H_t_d = torch.empty_like(x["H_s"]), torch.empty_like(x["H_t"])
-    mask_d, grad_d = torch.empty_like(mask), torch.empty_like(grad)
-    h2d = (H_s_h.numel() * H_s_h.element_size() + H_t_h.numel() * H_t_h.element_size() + mask_h.numel()
-           + grad_hp.numel() * 4)
-    d2h = kl_h.numel() * 4
+    # end to end through the same C ABI: the step's inputs from pinned host memory, its
+    # per-token result back to the host every step
+    host_in = {k: v.cpu().pin_memory() for k, v in inputs.items()}
+    dev_in = {k: torch.empty_like(v) for k, v in inputs.items()}
+    res_h = torch.empty(result.shape, dtype=result.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+    d2h = res_h.numel() * res_h.element_size()
 
     def e2e_step():
-        H_s_d.copy_(H_s_h, non_blocking=True)
-        H_t_d.copy_(H_t_h, non_blocking=True)
-        mask_d.copy_(mask_h, non_blocking=True)
-        grad_d.copy_(grad_hp, non_blocking=True)
-        step(H_s_d, H_t_d, mask_d, grad_d)
-        kl_h.copy_(kl, non_blocking=True)
+        for k, t in host_in.items():
+            dev_in[k].copy_(t, non_blocking=True)
+        step(dev_in)
+        res_h.copy_(result, non_blocking=True)
         torch.cuda.current_stream().synchronize()
-        return float(kl_h[0])
+        return float(res_h.view(-1)[0])
 
     e2e_step()
     barrier(world)
@@ -353,19 +448,18 @@ def run_gpu(args):
         return 0
 
     peaks, peak_src = load_peaks()
-    executed, algorithmic = step_flops(w, R)
     kernels = {}
     total_k = sum(v[1] for v in prof.values()) or 1.0
     for name, (n, tot) in sorted(prof.items(), key=lambda kv: -kv[1][1]):
         kernels[name] = {"launches": n, "ms_per_launch": tot / max(n, 1), "share": tot / total_k}
-    heavy = [k for k in kernels if kernel_flops(k, w, R) is not None]
+    heavy = [k for k in kernels if path_kernel_flops(args.path, k, w, R) is not None]
     dom = max(heavy, key=lambda k: kernels[k]["ms_per_launch"] * kernels[k]["launches"]) if heavy else None
     roofline = None
     if dom:
-        per_launch = kernel_flops(dom, w, R)
+        per_launch = path_kernel_flops(args.path, dom, w, R)
         achieved = per_launch / (kernels[dom]["ms_per_launch"] / 1000.0) / 1e12
         peak = peaks["bf16_tflops_sustained"]
-        traffic = recorded_traffic(dom, w.name)
+        traffic = recorded_traffic(dom, w.name) if args.path == "kl" else None
         roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak, "traffic": traffic,
                     "peak_source": f"bf16_tflops_sustained of {peak_src}",
@@ -374,18 +468,11 @@ def run_gpu(args):
 
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        host = host_inputs(x)
-        g = np.where(lay.mask != 0, grad_h.astype(np.float64), 0.0)
-        rows = sample_rows(lay.mask, args.cpu_rows, 3)
-        threads = os.cpu_count() or 1
-        rate, dt = oracle_rate(w, host, lay, g, rows, threads)
-        cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": f"{len(rows)} supervised rows of {w.name}: float64 logits, KL, dH_s rows and their "
-                         f"dW_s contribution ({dt:.1f} s)"}
+        cpu = path_cpu_baseline(args.path, w, lay, x, args)
 
     clocks = sampler.summary() if sampler else None
     out = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "metric": PATH_METRICS[args.path], "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded counter-based generator, packed multi-turn layout with masked observations "
@@ -403,6 +490,8 @@ def run_gpu(args):
         "clocks": clocks,
         "kernels": kernels,
     }
+    if args.path != "kl":
+        out["path"] = args.path
     print(json.dumps(out), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -468,6 +557,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--path", default="kl", choices=sorted(PATH_METRICS),
+                    help="kl: the reverse-KL step (default, the headline); surrogate: the sampled-token "
+                         "dual-clip surrogate; score: teacher token scoring")
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
     ap.add_argument("--ref-rows", type=int, default=8, help="rows per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
