@@ -272,7 +272,7 @@ def run_reference(args):
 
 PATH_METRICS = {
     "kl": METRIC,
-    "surrogate": "response tokens/s, sampled-token dual-clip surrogate fwd+bwd (1 GB300)",
+    "surrogate": "response tokens/s, sampled-token dual-clip surrogate loss step fwd+bwd (1 GB300)",
     "score": "response tokens/s, teacher token scoring fwd (1 GB300)",
 }
 
@@ -315,13 +315,20 @@ def path_setup(path, w, lay, x, dev, opd_kl):
     ws = opd_kl.allocate_workspace(prob, dev)
     loss, logp = torch.empty(w.T, device=dev), torch.empty(w.T, device=dev)
     dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+    n_ids = int(lay.seg_id.max()) + 1
+    seq_ws = torch.empty(opd_kl.opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8, device=dev)
+    dev_w = torch.empty(w.T, device=dev)
+    total = torch.empty(1, device=dev)
     inputs = {"H_s": x["H_s"], "tokens": tokens, "logp_old": logp_old, "logp_teacher": logp_teacher, "mask": mask,
-              "weights": weights}
+              "seg_id": torch.from_numpy(lay.seg_id).to(dev)}
 
     def step(i):
+        # weights on the device, the surrogate forward+backward, then the batch loss L
+        opd_kl.opd_seq_mean_token_mean_device(i["seg_id"], i["mask"], n_ids, 1e-8, None, dev_w, None, seq_ws)
         opd_kl.opd_surrogate_fwd_bwd(prob, i["H_s"], x["W_s"], i["tokens"], i["logp_old"], i["logp_teacher"],
-                                     i["mask"], i["weights"], loss, logp, dH, dW, False, ws)
-    return inputs, step, loss, ws, 8.0 * R * w.V * w.d_s, 6.0 * R * w.V * w.d_s
+                                     i["mask"], dev_w, loss, logp, dH, dW, False, ws)
+        opd_kl.opd_seq_mean_token_mean_device(i["seg_id"], i["mask"], n_ids, 1e-8, loss, None, total, seq_ws)
+    return inputs, step, total, ws, 8.0 * R * w.V * w.d_s, 6.0 * R * w.V * w.d_s
 
 
 def path_kernel_flops(path, name, w, R):

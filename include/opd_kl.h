@@ -177,9 +177,24 @@ opd_status opd_kl_forward_noalloc(const opd_problem* problem, const void* H_s, c
 opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t* mask, int64_t T, float eps,
                                            float* w_out);
 
+/* The same weights on the device, for a training step that stays on the GPU:
+ * seg_id [T] int32 and mask [T] uint8 in device memory, response ids in [0, n_ids) (ids < 0
+ * mark rows outside every response; an id >= n_ids sets the workspace status, reported as
+ * OPD_ERR_INVALID_ARG by opd_kl_get_status). Writes w_out [T] (device, may be NULL) and,
+ * when loss_in [T] and loss_out [1] are both given, loss_out[0] = sum_i w_i loss_in[i],
+ * which is the paper's L for per-token losses loss_in (accumulated in double; the
+ * summation order is not fixed). At least one of the two outputs must be requested.
+ * The workspace (device, 256-byte aligned) holds opd_seq_mean_token_mean_workspace_size(n_ids)
+ * bytes; it starts with the status word opd_kl_get_status reads. */
+size_t opd_seq_mean_token_mean_workspace_size(int64_t n_ids);
+opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* mask, int64_t T, int64_t n_ids,
+                                          float eps, const float* loss_in, float* w_out, float* loss_out,
+                                          void* workspace, size_t workspace_bytes, void* stream);
+
 /* Reads and clears the device status word in the workspace, after
  * synchronising the stream: OPD_OK, OPD_ERR_TIMEOUT if a bounded wait in the last
- * call ran out, or OPD_ERR_INVALID_ARG if a token id was outside [0, V). */
+ * call ran out, or OPD_ERR_INVALID_ARG if a token id was outside [0, V) (or a response
+ * id outside [0, n_ids) in opd_seq_mean_token_mean_device). */
 opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stream);
 
 /* Self-test of the bounded-wait machinery: launches one kernel that waits on a

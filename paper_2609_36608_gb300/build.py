@@ -21,7 +21,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libopdkl.so")
 
 SOURCES = ["opd_api.cu", "opd_aux.cu", "opd_simt.cu", "opd_fused.cu", "opd_gemm.cu", "opd_noalloc.cu",
-           "opd_surrogate.cu"]
+           "opd_surrogate.cu", "opd_seqmean.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -549,6 +549,32 @@ opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t*
   return OPD_OK;
 }
 
+size_t opd_seq_mean_token_mean_workspace_size(int64_t n_ids) {
+  if (n_ids < 1 || n_ids > (int64_t)0x7FFF0000) return 0;
+  return round_up(seq_mean_token_mean_scratch_bytes(n_ids), 256);
+}
+
+opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* mask, int64_t T, int64_t n_ids,
+                                          float eps, const float* loss_in, float* w_out, float* loss_out,
+                                          void* workspace, size_t workspace_bytes, void* stream) {
+  if (T < 0 || T > (int64_t)0x7FFF0000 || n_ids < 1 || n_ids > (int64_t)0x7FFF0000 || !(eps >= 0.0f))
+    return OPD_ERR_INVALID_ARG;
+  if (T > 0 && (!seg_id || !mask)) return OPD_ERR_INVALID_ARG;
+  if (!w_out && !(loss_in && loss_out)) return OPD_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < opd_seq_mean_token_mean_workspace_size(n_ids))
+    return OPD_ERR_INVALID_ARG;
+  const DeviceInfo dev = device_info();
+  if (dev.sm_count <= 0) return OPD_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  OPD_CUDA(timed("seq_mean_token_mean", s, [&] {
+    return launch_seq_mean_token_mean(seg_id, mask, (int32_t)T, (int32_t)n_ids, eps, loss_in, w_out,
+                                      loss_in ? loss_out : nullptr, workspace, dev.sm_count, s);
+  }));
+  if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
+  if (env_flag("OPD_KL_SYNC_CHECK")) return opd_kl_get_status(workspace, workspace_bytes, stream);
+  return OPD_OK;
+}
+
 opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stream) {
   if (!workspace || workspace_bytes < sizeof(Ctrl) || !aligned(workspace, 256)) return OPD_ERR_INVALID_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -112,6 +112,11 @@ cudaError_t launch_head_forward(const CUtensorMap& h, const CUtensorMap& w, cons
 cudaError_t launch_head_backward(const CUtensorMap& h, const CUtensorMap& w, const CUtensorMap& dz_store,
                                  const FusedParams& p, int grid, cudaStream_t s);
 cudaError_t launch_head_rows(const HeadRowsParams& p, int n_sm, cudaStream_t s);
+// seq-mean-token-mean on the device (opd_seqmean.cu); workspace starts with a Ctrl.
+size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids);
+cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, float eps,
+                                       const float* loss_in, float* w_out, float* loss_out, void* workspace,
+                                       int n_sm, cudaStream_t s);
 // C = A * B^T with A [M, K] and B [N, K] given through tensor maps; a_mn / b_mn select
 // MN-major operand tiles (the operand's contiguous dimension is M or N, not K).
 cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,

@@ -1,0 +1,99 @@
+// seq-mean-token-mean on the device (ActFirst-OPD Appendix B.4, Eq. opd-surrogate):
+//   L = 1/|B| sum_b ( sum_j m_bj l_bj ) / ( sum_j m_bj + eps )
+// so the weight of token i is w_i = m_i / (|B| (n_seg(i) + eps)), with n_b the number of
+// supervised tokens of response b and |B| the number of distinct responses (ids >= 0,
+// including responses whose tokens are all masked). Three small memory-bound passes:
+// a histogram of supervised tokens per response id, the count of distinct ids, then the
+// weights and (optionally) sum_i w_i l_i.
+#include "opd_device.cuh"
+#include "opd_internal.h"
+
+namespace opd {
+
+namespace {
+
+// Workspace: Ctrl (status), then [double acc][int32 n_resp, pad][counts n_ids][present n_ids].
+__global__ void k_seq_zero(Ctrl* ctrl, int32_t* counts, int32_t* present, int32_t n_ids, int32_t* n_resp,
+                           double* acc) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_ids; i += gridDim.x * blockDim.x) {
+    counts[i] = 0;
+    present[i] = 0;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    ctrl->status = 0u;
+    *n_resp = 0;
+    *acc = 0.0;
+  }
+}
+
+__global__ void k_seq_hist(const int32_t* __restrict__ seg, const uint8_t* __restrict__ mask, int32_t T,
+                           int32_t n_ids, int32_t* counts, int32_t* present, uint32_t* status) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+    const int b = seg[i];
+    if (b < 0) continue;
+    if (b >= n_ids) {
+      atomicOr(status, kDevBadToken);
+      continue;
+    }
+    present[b] = 1;
+    if (mask[i]) atomicAdd(&counts[b], 1);
+  }
+}
+
+__global__ void k_seq_count(const int32_t* __restrict__ present, int32_t n_ids, int32_t* n_resp) {
+  int local = 0;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_ids; i += gridDim.x * blockDim.x) local += present[i];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) local += __shfl_xor_sync(0xffffffffu, local, o);
+  if ((threadIdx.x & 31) == 0 && local) atomicAdd(n_resp, local);
+}
+
+__global__ void k_seq_weights(const int32_t* __restrict__ seg, const uint8_t* __restrict__ mask, int32_t T,
+                              int32_t n_ids, const int32_t* __restrict__ counts, const int32_t* __restrict__ n_resp,
+                              float eps, const float* __restrict__ loss_in, float* __restrict__ w_out, double* acc) {
+  const double nb = (double)*n_resp;
+  double part = 0.0;
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+    const int b = seg[i];
+    float w = 0.f;
+    if (b >= 0 && b < n_ids && mask[i]) w = (float)(1.0 / (nb * ((double)counts[b] + (double)eps)));
+    if (w_out) w_out[i] = w;
+    if (loss_in) part += (double)w * (double)loss_in[i];
+  }
+  if (loss_in) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    if ((threadIdx.x & 31) == 0 && part != 0.0) atomicAdd(acc, part);
+  }
+}
+
+__global__ void k_seq_store(const double* acc, float* loss_out) { *loss_out = (float)*acc; }
+
+}  // namespace
+
+size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids) { return sizeof(Ctrl) + 16 + 8 * (size_t)n_ids; }
+
+cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, float eps,
+                                       const float* loss_in, float* w_out, float* loss_out, void* workspace,
+                                       int n_sm, cudaStream_t s) {
+  Ctrl* ctrl = static_cast<Ctrl*>(workspace);
+  double* acc = reinterpret_cast<double*>(static_cast<uint8_t*>(workspace) + sizeof(Ctrl));
+  int32_t* n_resp = reinterpret_cast<int32_t*>(acc + 1);
+  int32_t* counts = n_resp + 2;
+  int32_t* present = counts + n_ids;
+  uint32_t* status = &ctrl->status;
+  const int threads = 256;
+  auto blocks = [&](long work) {
+    long b = (work + threads - 1) / threads;
+    if (b > (long)n_sm * 4) b = (long)n_sm * 4;
+    return (int)(b < 1 ? 1 : b);
+  };
+  k_seq_zero<<<blocks(n_ids), threads, 0, s>>>(ctrl, counts, present, n_ids, n_resp, acc);
+  k_seq_hist<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, present, status);
+  k_seq_count<<<blocks(n_ids), threads, 0, s>>>(present, n_ids, n_resp);
+  k_seq_weights<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, n_resp, eps, loss_in, w_out, acc);
+  if (loss_out) k_seq_store<<<1, 1, 0, s>>>(acc, loss_out);
+  return cudaGetLastError();
+}
+
+}  // namespace opd

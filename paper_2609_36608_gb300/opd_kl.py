@@ -69,6 +69,8 @@ def _load() -> ctypes.CDLL:
         "opd_score_tokens": (i32, [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
         "opd_surrogate_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, vp, ctypes.POINTER(opd_surrogate_params),
                                         vp, vp, vp, vp, i32, vp, sz, vp]),
+        "opd_seq_mean_token_mean_workspace_size": (sz, [i64]),
+        "opd_seq_mean_token_mean_device": (i32, [vp, vp, i64, i64, ctypes.c_float, vp, vp, vp, vp, sz, vp]),
         "opd_kl_profile_start": (i32, []),
         "opd_kl_profile_stop": (i32, [ctypes.POINTER(opd_kernel_time), i32, ctypes.POINTER(i32)]),
     }
@@ -184,6 +186,24 @@ def opd_seq_mean_token_mean_weights(seg_id, mask, eps: float = 1e-8) -> np.ndarr
                                                 s.shape[0], float(eps), w.ctypes.data_as(ctypes.c_void_p)),
            "opd_seq_mean_token_mean_weights")
     return w
+
+
+def opd_seq_mean_token_mean_workspace_size(n_ids: int) -> int:
+    return int(_lib.opd_seq_mean_token_mean_workspace_size(int(n_ids)))
+
+
+def opd_seq_mean_token_mean_device(seg_id, mask, n_ids: int, eps: float = 1e-8, loss_in=None, w_out=None,
+                                   loss_out=None, workspace=None, stream=None) -> torch.Tensor:
+    """seq-mean-token-mean weights (and optionally the weighted loss) on the device; returns the
+    workspace used (its status word is what opd_kl_get_status reads)."""
+    if workspace is None:
+        workspace = torch.empty(opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8,
+                                device=seg_id.device)
+    _check(_lib.opd_seq_mean_token_mean_device(_ptr(seg_id), _ptr(mask), seg_id.numel(), int(n_ids), float(eps),
+                                               _ptr(loss_in), _ptr(w_out), _ptr(loss_out), _ptr(workspace),
+                                               workspace.numel(), _stream(stream)),
+           "opd_seq_mean_token_mean_device")
+    return workspace
 
 
 def opd_kl_get_status(workspace, stream=None) -> int:

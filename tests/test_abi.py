@@ -88,3 +88,21 @@ def test_seq_mean_token_mean_helper_matches_oracle(lib, oracle_mod):
         np.testing.assert_allclose(w, ref, rtol=2e-7, atol=0)
     with pytest.raises(lib.OpdError):
         lib.opd_seq_mean_token_mean_weights(np.zeros(3, np.int32), np.zeros(3, np.uint8), -1.0)
+
+
+def test_seq_mean_token_mean_device_arguments(lib):
+    assert lib.opd_seq_mean_token_mean_workspace_size(0) == 0
+    assert lib.opd_seq_mean_token_mean_workspace_size(100) >= 256 + 16 + 800
+    vp = ctypes.c_void_p
+    fake = vp(1 << 20)
+    # no output requested
+    rc = lib.call_raw("opd_seq_mean_token_mean_device", fake, fake, ctypes.c_int64(4), ctypes.c_int64(2),
+                      ctypes.c_float(1e-8), None, None, None, fake, ctypes.c_size_t(4096), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+    # workspace too small
+    rc = lib.call_raw("opd_seq_mean_token_mean_device", fake, fake, ctypes.c_int64(4), ctypes.c_int64(1000),
+                      ctypes.c_float(1e-8), None, fake, None, fake, ctypes.c_size_t(512), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+    rc = lib.call_raw("opd_seq_mean_token_mean_device", fake, fake, ctypes.c_int64(4), ctypes.c_int64(2),
+                      ctypes.c_float(-1.0), None, fake, None, fake, ctypes.c_size_t(4096), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
