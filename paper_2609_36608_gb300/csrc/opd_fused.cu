@@ -18,11 +18,12 @@
 // tile, vocabulary range) are walked grid-strided.
 //
 // TMEM holds one tile: teacher accumulator in columns [0,256), student in
-// [256,512). Each tile computes the teacher segment first. The epilogue copies
-// its teacher columns to registers and releases them at once, so the next tile's
-// teacher GEMM (d_t of the d_s + d_t reduction) overlaps this tile's epilogue;
-// the student columns are released as soon as they have been read, well before
-// the next tile's student GEMM starts.
+// [256,512). Each tile computes the teacher segment first and signals it on its
+// own barrier. While the student segment runs, the epilogue copies the teacher
+// columns to registers and releases them, so the next tile's teacher GEMM (d_t of
+// the d_s + d_t reduction) follows this tile's student GEMM without a gap and
+// overlaps this tile's epilogue; the student columns are released as soon as they
+// have been read, well before the next tile's student GEMM starts.
 //
 // PAIR = true runs each tile on a CTA pair (2-CTA cluster, tcgen05 cta_group::2):
 // 256 rows per tile, 128 in each CTA's TMEM; each CTA stages its own 128 rows of
@@ -260,9 +261,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   float* merge = reinterpret_cast<float*>(staging + kNEpi * C::kStagingPerWarp);
   uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(merge) + C::kMergeBytes);
   uint64_t* empty = full + C::kStages;
-  // acc_full[0]: both segments of a tile computed (two heads). One head: acc_full[slot]
-  // for TMEM slot 0 / 1 (columns 0-255 / 256-511, alternate tiles), so each barrier runs
-  // at most one phase ahead of the epilogue that waits on it.
+  // Two heads: acc_full[1] completes when a tile's teacher segment is computed,
+  // acc_full[0] when its student segment is. One head: acc_full[slot] for TMEM slot 0 / 1
+  // (columns 0-255 / 256-511, alternate tiles). Each barrier runs at most one phase ahead
+  // of the epilogue that waits on it.
   uint64_t* acc_full = empty + C::kStages;
   // Two heads: teacher / student columns read by every epilogue warp. One head: slot 0 /
   // slot 1 read by every epilogue warp.
@@ -430,6 +432,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 phase ^= 1u;
               }
             }
+            // two heads: the teacher segment is signalled on its own, so the epilogue
+            // can drain and release its columns while the student segment runs
+            if (HEADS == 2 && seg == 0 && ok) {
+              if (PAIR)
+                umma_commit_pair_mc(&acc_full[1], 0x3);
+              else
+                umma_commit(&acc_full[1]);
+            }
           }
           if (ok) {
             uint64_t* af = HEADS == 2 ? &acc_full[0] : &acc_full[lt & 1];
@@ -483,8 +493,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       for (int vt = vb; vt < ve; ++vt, ++lt) {
-        // warp-uniform outcome: the TMEM loads below are .sync.aligned
-        uint64_t* af = HEADS == 2 ? &acc_full[0] : &acc_full[lt & 1];
+        // warp-uniform outcome: the TMEM loads below are .sync.aligned. Two heads wait
+        // first for the teacher segment (acc_full[1]), one head for its slot's tile.
+        uint64_t* af = HEADS == 2 ? &acc_full[1] : &acc_full[lt & 1];
         const uint32_t af_par = HEADS == 2 ? ((uint32_t)lt & 1u) : (((uint32_t)lt >> 1) & 1u);
         if (!__all_sync(0xffffffffu, mbar_wait(af, af_par, status, lim))) {
           ok = false;
@@ -546,6 +557,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           else
             mbar_arrive(t_free);
         }
+        // then the student segment (committed after the teacher's, same tile parity)
+        if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[0], (uint32_t)lt & 1u, status, lim))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
         const int col0 = vt * kBN + cbase;
         const uint32_t ts = tmem_s + t_lane + (uint32_t)cbase;
         if (!BWD) {
