@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(kCompactThreads)
   __shared__ int32_t warp_tot[32];
   const int tid = threadIdx.x;
   if (tid == 0) ctrl->status = 0u;
+  if (tid < 4) ctrl->work[tid] = 0;
   const int per = (T + kCompactThreads - 1) / kCompactThreads;
   const int lo = min(T, tid * per);
   const int hi = min(T, lo + per);

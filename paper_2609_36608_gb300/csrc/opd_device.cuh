@@ -23,7 +23,8 @@ struct Ctrl {
   int32_t R;          // supervised rows (written by the compaction kernel)
   uint32_t status;    // kDev* bits, cleared at the start of every call
   int32_t n_vsplit;   // vocabulary splits the forward used (written by the fused forward)
-  int32_t pad[61];
+  int32_t work[4];    // work-unit counters of the fused kernels, zeroed at the start of every call
+  int32_t pad[57];
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -67,17 +68,33 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t addr, uint32_t parity) {
   return ok != 0;
 }
 
+// Cluster-scope acquire: also orders what another CTA of the cluster wrote into
+// this CTA's shared memory before its release-arrive on the barrier.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Wait until the phase of the given parity has completed. Every wait is bounded:
 // after limit_ns of wall time (or 2^30 polls) it flags kDevTimeout in the status
 // word and returns false; it also gives up early once any other thread of the
 // grid has flagged an error, so one failure unwinds every role quickly.
+template <bool CLUSTER = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t* status,
                                           uint64_t limit_ns) {
   const uint32_t addr = smem_u32(bar);
-  if (mbar_try_wait(addr, parity)) return true;
+  auto poll = [&] { return CLUSTER ? mbar_try_wait_cluster(addr, parity) : mbar_try_wait(addr, parity); };
+  if (poll()) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(addr, parity)) return true;
+    if (poll()) return true;
     if ((it & 63u) == 0) {
       if (*reinterpret_cast<volatile uint32_t*>(status) != 0u) return false;
       if (globaltimer_ns() - t0 > limit_ns || it >= (1u << 30)) {
@@ -237,6 +254,10 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t smem_addr, uint32_t ran
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
   return r;
+}
+
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {

@@ -41,6 +41,7 @@ constexpr int kBN = 256;   // vocabulary columns per tile (MMA N)
 constexpr int kNEpi = 8;   // epilogue warps
 constexpr int kColsPerWarp = kBN / 2;
 constexpr int kThreads = 64 + 32 * kNEpi;
+constexpr int kUnitRing = 8;  // work-unit indices in flight between the fetching thread and the other roles
 
 template <bool BWD, bool PAIR, int HEADS>
 struct FusedCfg {
@@ -51,7 +52,7 @@ struct FusedCfg {
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
   static constexpr uint32_t kStagingPerWarp = BWD ? 32 * kColsPerWarp * 2 : 0;  // bf16 dz rows of one warp
   static constexpr uint32_t kMergeBytes = BWD ? 0 : 4 * 5 * 32 * 4;             // per quadrant 5 x 32
-  static constexpr uint32_t kBarrierBytes = 256;
+  static constexpr uint32_t kBarrierBytes = 512;
   static constexpr size_t kFixed = 1024 + (size_t)kNEpi * kStagingPerWarp + kMergeBytes + kBarrierBytes;
   static constexpr int kStagesFit = (int)((232448 - kFixed) / kStageBytes);
   static constexpr int kStages = kStagesFit > 8 ? 8 : kStagesFit;
@@ -63,7 +64,9 @@ struct FusedCfg {
 
 // Unit u -> (row tile, vocabulary tile range). Units are grouped by `G` row tiles
 // so that CTAs (or CTA pairs) running at the same time share a few hidden-state
-// tiles and a few vocabulary tiles in L2.
+// tiles and a few vocabulary tiles in L2. Workers take units in increasing order
+// from a global counter (not a fixed stride), so the workers that share a
+// vocabulary range start it together and stay together however their speeds differ.
 struct FusedSchedule {
   int n_rt, n_vt, n_vs, G, n_units;
 
@@ -248,6 +251,56 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
                  w[4 * jj + 3]);
 }
 
+// Work-unit ring. One thread (the producer of the pair's even CTA) takes unit
+// indices from the global counter and publishes each in both CTAs' rings; the MMA
+// issuer, the epilogue warps and the odd CTA's producer read them in the same
+// order and release the slot. Returns the k-th unit, or -1 if a wait failed.
+template <bool PAIR>
+__device__ __forceinline__ int fetch_unit(uint32_t k, int32_t* counter, uint64_t* unit_full, uint64_t* unit_empty,
+                                          int32_t* units, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!mbar_wait<true>(&unit_empty[slot], par ^ 1u, status, lim)) return -1;
+  const int u = atomicAdd(counter, 1);
+  units[slot] = u;
+  if (PAIR) {
+    st_shared_cluster_u32(mapa_shared(smem_u32(&units[slot]), 1u), (uint32_t)u);
+    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_full[slot]), 1u));
+  }
+  mbar_arrive(&unit_full[slot]);
+  return u;
+}
+
+// Reader side, one thread. `remote`: release the slot in the pair's even CTA.
+template <bool PAIR>
+__device__ __forceinline__ int take_unit(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty, const int32_t* units,
+                                         bool remote, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!mbar_wait<PAIR>(&unit_full[slot], par, status, lim)) return -1;
+  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
+  if (remote)
+    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
+  else
+    mbar_arrive(&unit_empty[slot]);
+  return u;
+}
+
+// Reader side, one warp (warp-uniform result; lane 0 releases the slot).
+template <bool PAIR>
+__device__ __forceinline__ int take_unit_warp(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty,
+                                              const int32_t* units, bool remote, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!__all_sync(0xffffffffu, mbar_wait<PAIR>(&unit_full[slot], par, status, lim))) return -1;
+  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) {
+    if (remote)
+      mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
+    else
+      mbar_arrive(&unit_empty[slot]);
+  }
+  return u;
+}
+
 template <bool BWD, bool PAIR, int HEADS>
 __global__ void __launch_bounds__(kThreads, 1)
     k_fused_logits(const __grid_constant__ CUtensorMap tm_hs, const __grid_constant__ CUtensorMap tm_ht,
@@ -273,15 +326,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* mma_done = s_free + 1;
   uint64_t* merge_full = mma_done + 1;      // [4]
   uint64_t* merge_empty = merge_full + 4;   // [4]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(merge_empty + 4);
+  uint64_t* unit_full = merge_empty + 4;    // [kUnitRing]
+  uint64_t* unit_empty = unit_full + kUnitRing;
+  int32_t* units = reinterpret_cast<int32_t*>(unit_empty + kUnitRing);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(units + kUnitRing);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   uint32_t* status = &p.ctrl->status;
   const uint64_t lim = p.wait_limit_ns;
   const uint32_t rank = PAIR ? cluster_ctarank() : 0u;  // CTA rank within the pair
-  const int worker = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
   const int n_workers = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  int32_t* counter = &p.ctrl->work[BWD ? 1 : 0];
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
@@ -296,6 +352,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int qd = 0; qd < 4; ++qd) {
       mbar_init(&merge_full[qd], 1);
       mbar_init(&merge_empty[qd], 1);
+    }
+    // readers of each ring slot: the MMA issuer and the epilogue warps of the even
+    // CTA, plus the odd CTA's producer and epilogue warps in a pair
+    for (int i = 0; i < kUnitRing; ++i) {
+      mbar_init(&unit_full[i], 1);
+      mbar_init(&unit_empty[i], PAIR ? 2 * (1 + kNEpi) : 1 + kNEpi);
     }
     fence_mbar_init();
   }
@@ -339,7 +401,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true, any = false;
       // a pair counts both CTAs' bytes on the leader's full barriers
       const uint32_t full_leader = PAIR ? mapa_shared(smem_u32(full), 0u) : smem_u32(full);
-      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
+      for (uint32_t k = 0; ok; ++k) {
+        const int u = rank == 0 ? fetch_unit<PAIR>(k, counter, unit_full, unit_empty, units, status, lim)
+                                : take_unit<PAIR>(k, unit_full, unit_empty, units, true, status, lim);
+        if (u < 0) {
+          ok = false;
+          break;
+        }
+        if (u >= sch.n_units) break;
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
         const int row0 = rt * C::kTileRows + (int)rank * kRowTile;
@@ -390,7 +459,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
-      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
+      for (uint32_t k = 0; ok; ++k) {
+        const int u = take_unit<PAIR>(k, unit_full, unit_empty, units, false, status, lim);
+        if (u < 0) {
+          ok = false;
+          break;
+        }
+        if (u >= sch.n_units) break;
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
         for (int vt = vb; ok && vt < ve; ++vt, ++lt) {
@@ -471,7 +546,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     int lt = 0, nu = 0;
     bool ok = true;
     const uint32_t stg = smem_u32(staging + ew * C::kStagingPerWarp);
-    for (int u = worker; ok && u < sch.n_units; u += n_workers, ++nu) {
+    for (uint32_t k = 0; ok; ++k, ++nu) {
+      const int u = take_unit_warp<PAIR>(k, unit_full, unit_empty, units, PAIR && rank != 0, status, lim);
+      if (u < 0) {
+        ok = false;
+        break;
+      }
+      if (u >= sch.n_units) break;
       int rt, split, vb, ve;
       sch.unit(u, rt, split, vb, ve);
       const int row_base = rt * C::kTileRows + (int)rank * kRowTile;

@@ -50,6 +50,7 @@ __global__ void k_noalloc_rows(const uint8_t* __restrict__ mask, int32_t T) {
     ctrl->status = 0u;
     ctrl->n_vsplit = 0;
   }
+  if (threadIdx.x < 4) ctrl->work[threadIdx.x] = 0;
 }
 
 // Device address of the scratch array, looked up once per device (with that
