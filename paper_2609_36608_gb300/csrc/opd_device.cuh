@@ -23,7 +23,7 @@ struct Ctrl {
   int32_t R;          // supervised rows (written by the compaction kernel)
   uint32_t status;    // kDev* bits, cleared at the start of every call
   int32_t n_vsplit;   // vocabulary splits the forward used (written by the fused forward)
-  int32_t work[4];    // work-unit counters of the fused kernels, zeroed at the start of every call
+  int32_t work[4];    // work-unit counters of the fused kernels (forward, backward), zeroed per call
   int32_t pad[57];
 };
 
@@ -333,6 +333,62 @@ __device__ __forceinline__ uint32_t sw128_offset(uint32_t r, uint32_t j) {
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+constexpr int kUnitRing = 8;  // unit indices in flight between the fetching thread and the readers
+
+// ------------------------------------------------------------ work units --
+//
+// Persistent kernels take work units in increasing order from a global counter
+// (Ctrl::work). One thread per CTA (per pair: the even CTA's producer) claims
+// each index one unit ahead of its use (hiding the atomic's latency) and
+// publishes it in a ring of kUnitRing slots, in both CTAs of a pair; every other
+// role reads the same sequence and releases each slot (the slot's empty barrier
+// counts all readers). publish_unit returns false if a wait failed.
+template <bool PAIR>
+__device__ __forceinline__ bool publish_unit(uint32_t k, int u, uint64_t* unit_full, uint64_t* unit_empty,
+                                             int32_t* units, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!mbar_wait<true>(&unit_empty[slot], par ^ 1u, status, lim)) return false;
+  units[slot] = u;
+  if (PAIR) {
+    st_shared_cluster_u32(mapa_shared(smem_u32(&units[slot]), 1u), (uint32_t)u);
+    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_full[slot]), 1u));
+  }
+  mbar_arrive(&unit_full[slot]);
+  return true;
+}
+
+// Reader side, one thread: the k-th unit, or -1 if the wait failed. `remote`:
+// release the slot in the pair's even CTA.
+template <bool PAIR>
+__device__ __forceinline__ int take_unit(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty, const int32_t* units,
+                                         bool remote, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!mbar_wait<PAIR>(&unit_full[slot], par, status, lim)) return -1;
+  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
+  if (remote)
+    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
+  else
+    mbar_arrive(&unit_empty[slot]);
+  return u;
+}
+
+// Reader side, one warp (warp-uniform result; lane 0 releases the slot).
+template <bool PAIR>
+__device__ __forceinline__ int take_unit_warp(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty,
+                                              const int32_t* units, bool remote, uint32_t* status, uint64_t lim) {
+  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
+  if (!__all_sync(0xffffffffu, mbar_wait<PAIR>(&unit_full[slot], par, status, lim))) return -1;
+  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) {
+    if (remote)
+      mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
+    else
+      mbar_arrive(&unit_empty[slot]);
+  }
+  return u;
 }
 
 }  // namespace opd

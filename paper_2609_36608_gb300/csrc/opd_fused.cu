@@ -41,7 +41,6 @@ constexpr int kBN = 256;   // vocabulary columns per tile (MMA N)
 constexpr int kNEpi = 8;   // epilogue warps
 constexpr int kColsPerWarp = kBN / 2;
 constexpr int kThreads = 64 + 32 * kNEpi;
-constexpr int kUnitRing = 8;  // work-unit indices in flight between the fetching thread and the other roles
 
 template <bool BWD, bool PAIR, int HEADS>
 struct FusedCfg {
@@ -251,56 +250,6 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
                  w[4 * jj + 3]);
 }
 
-// Work-unit ring. One thread (the producer of the pair's even CTA) takes unit
-// indices from the global counter and publishes each in both CTAs' rings; the MMA
-// issuer, the epilogue warps and the odd CTA's producer read them in the same
-// order and release the slot. Returns the k-th unit, or -1 if a wait failed.
-template <bool PAIR>
-__device__ __forceinline__ int fetch_unit(uint32_t k, int32_t* counter, uint64_t* unit_full, uint64_t* unit_empty,
-                                          int32_t* units, uint32_t* status, uint64_t lim) {
-  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
-  if (!mbar_wait<true>(&unit_empty[slot], par ^ 1u, status, lim)) return -1;
-  const int u = atomicAdd(counter, 1);
-  units[slot] = u;
-  if (PAIR) {
-    st_shared_cluster_u32(mapa_shared(smem_u32(&units[slot]), 1u), (uint32_t)u);
-    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_full[slot]), 1u));
-  }
-  mbar_arrive(&unit_full[slot]);
-  return u;
-}
-
-// Reader side, one thread. `remote`: release the slot in the pair's even CTA.
-template <bool PAIR>
-__device__ __forceinline__ int take_unit(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty, const int32_t* units,
-                                         bool remote, uint32_t* status, uint64_t lim) {
-  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
-  if (!mbar_wait<PAIR>(&unit_full[slot], par, status, lim)) return -1;
-  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
-  if (remote)
-    mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
-  else
-    mbar_arrive(&unit_empty[slot]);
-  return u;
-}
-
-// Reader side, one warp (warp-uniform result; lane 0 releases the slot).
-template <bool PAIR>
-__device__ __forceinline__ int take_unit_warp(uint32_t k, uint64_t* unit_full, uint64_t* unit_empty,
-                                              const int32_t* units, bool remote, uint32_t* status, uint64_t lim) {
-  const uint32_t slot = k & (kUnitRing - 1), par = (k / kUnitRing) & 1u;
-  if (!__all_sync(0xffffffffu, mbar_wait<PAIR>(&unit_full[slot], par, status, lim))) return -1;
-  const int u = *reinterpret_cast<const volatile int32_t*>(&units[slot]);
-  __syncwarp();
-  if ((threadIdx.x & 31) == 0) {
-    if (remote)
-      mbar_arrive_cluster(mapa_shared(smem_u32(&unit_empty[slot]), 0u));
-    else
-      mbar_arrive(&unit_empty[slot]);
-  }
-  return u;
-}
-
 template <bool BWD, bool PAIR, int HEADS>
 __global__ void __launch_bounds__(kThreads, 1)
     k_fused_logits(const __grid_constant__ CUtensorMap tm_hs, const __grid_constant__ CUtensorMap tm_ht,
@@ -401,9 +350,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true, any = false;
       // a pair counts both CTAs' bytes on the leader's full barriers
       const uint32_t full_leader = PAIR ? mapa_shared(smem_u32(full), 0u) : smem_u32(full);
+      int next = rank == 0 ? atomicAdd(counter, 1) : 0;
       for (uint32_t k = 0; ok; ++k) {
-        const int u = rank == 0 ? fetch_unit<PAIR>(k, counter, unit_full, unit_empty, units, status, lim)
-                                : take_unit<PAIR>(k, unit_full, unit_empty, units, true, status, lim);
+        int u = -1;
+        if (rank == 0) {
+          u = next;
+          if (!publish_unit<PAIR>(k, u, unit_full, unit_empty, units, status, lim)) u = -1;
+          if (u >= 0 && u < sch.n_units) next = atomicAdd(counter, 1);  // used by the next iteration
+        } else {
+          u = take_unit<PAIR>(k, unit_full, unit_empty, units, true, status, lim);
+        }
         if (u < 0) {
           ok = false;
           break;
