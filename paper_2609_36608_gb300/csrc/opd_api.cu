@@ -261,6 +261,12 @@ struct Maps {
   CUtensorMap dz_a_mn, hsg_b_mn, dw; // dW_s GEMM
 };
 
+// Gradient-GEMM tiling: CTA pairs unless OPD_KL_GEMM=cta1.
+int gemm_pair_mode() {
+  const char* v = std::getenv("OPD_KL_GEMM");
+  return (v && std::strcmp(v, "cta1") == 0) ? 0 : 1;
+}
+
 // Fused-kernel tiling: OPD_KL_FUSED=bn256 | pair256 overrides the default.
 int fused_tile_mode() {
   const char* v = std::getenv("OPD_KL_FUSED");
@@ -353,6 +359,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s
   gh.k_is_R = 0;
   gh.max_ksplit = env_int("OPD_KL_MAX_KSPLIT", kMaxKSplit);
   gh.reduce = 1;
+  gh.pair = gemm_pair_mode();
   gh.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dH", c.s, [&] { return launch_gemm(false, true, m.dz_a_k, m.ws_b_mn, m.dhg, gh, c.dev.sm_count, c.s); }));
 
@@ -365,6 +372,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s
   gw.k_is_R = 1;
   gw.max_ksplit = 1;
   gw.reduce = accumulate_dW ? 1 : 0;
+  gw.pair = gemm_pair_mode();
   gw.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dW", c.s, [&] { return launch_gemm(true, true, m.dz_a_mn, m.hsg_b_mn, m.dw, gw, c.dev.sm_count, c.s); }));
 

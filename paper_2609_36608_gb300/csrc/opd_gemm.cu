@@ -11,6 +11,11 @@
 // K blocks staged by TMA with 128-byte swizzle, one thread issuing MMAs, four
 // epilogue warps draining TMEM through swizzled shared memory into TMA stores
 // (or TMA reduce-adds, for split-K partial sums and for accumulating into dW_s).
+//
+// PAIR = true runs 256 x 256 tiles on a CTA pair (tcgen05 cta_group::2): each CTA
+// stages its own 128 rows of A and 128 of the 256 columns of B, holds its 128 x 256
+// accumulator in its own TMEM and stores it; the even CTA issues the MMAs. Per
+// byte staged from L2 this does 1.5 times the MMA work of the single-CTA tile.
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
@@ -19,20 +24,28 @@ namespace opd {
 namespace {
 
 constexpr int kBN = kGemmBN;
-constexpr int kStages = 4;
-constexpr uint32_t kABytes = kRowTile * kKBlock * 2;  // 16 KB
-constexpr uint32_t kBBytes = kBN * kKBlock * 2;       // 32 KB
-constexpr uint32_t kStageBytes = kABytes + kBBytes;
 constexpr uint32_t kChunkBytes = 32 * 32 * 4;         // one 32x32 fp32 staging box
 constexpr uint32_t kStagingPerWarp = 2 * kChunkBytes;
-constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + 4 * kStagingPerWarp + 256;
-static_assert(kSmem <= 232448, "shared memory budget");
+
+template <bool PAIR>
+struct GemmCfg {
+  static constexpr int kTileRows = PAIR ? 2 * kRowTile : kRowTile;  // M rows per tile (whole pair)
+  static constexpr int kBCols = PAIR ? kBN / 2 : kBN;               // N columns of B one CTA stages
+  static constexpr uint32_t kABytes = kRowTile * kKBlock * 2;       // 16 KB
+  static constexpr uint32_t kBBytes = kBCols * kKBlock * 2;         // 32 KB (16 KB in a pair)
+  static constexpr uint32_t kStageBytes = kABytes + kBBytes;
+  static constexpr size_t kFixed = 1024 + 4 * kStagingPerWarp + 256;
+  static constexpr int kStages = (int)((232448 - kFixed) / kStageBytes) > 6 ? 6 : (int)((232448 - kFixed) / kStageBytes);
+  static constexpr size_t kSmem = kFixed + (size_t)kStages * kStageBytes;
+  static_assert(kStages >= 4, "pipeline depth");
+  static_assert(kSmem <= 232448, "shared memory budget");
+};
 
 struct GemmSchedule {
   int n_mt, n_nt, nkb, n_ks, n_units;
 
-  __device__ void init(int M, int N, int K, int grid, int max_ks) {
-    n_mt = (M + kRowTile - 1) / kRowTile;
+  __device__ void init(int M, int N, int K, int tile_rows, int grid, int max_ks) {
+    n_mt = (M + tile_rows - 1) / tile_rows;
     n_nt = (N + kBN - 1) / kBN;
     nkb = (K + kKBlock - 1) / kKBlock;
     n_ks = 1;
@@ -73,10 +86,14 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, 
   }
 }
 
-template <bool A_MN, bool B_MN>
+template <bool A_MN, bool B_MN, bool PAIR>
 __global__ void __launch_bounds__(192, 1)
     k_umma_gemm(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
                 const __grid_constant__ CUtensorMap tm_c, const GemmParams p) {
+  using C = GemmCfg<PAIR>;
+  constexpr int kStages = C::kStages;
+  constexpr uint32_t kABytes = C::kABytes;
+  constexpr uint32_t kStageBytes = C::kStageBytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* stage_base = smem;
@@ -92,6 +109,9 @@ __global__ void __launch_bounds__(192, 1)
   const int lane = threadIdx.x & 31;
   uint32_t* status = &p.ctrl->status;
   const uint64_t lim = p.wait_limit_ns;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;  // CTA rank within the pair
+  const int worker = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int n_workers = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -100,7 +120,7 @@ __global__ void __launch_bounds__(192, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], 4);
+      mbar_init(&acc_empty[b], PAIR ? 8 : 4);  // epilogue warps of the pair
     }
     mbar_init(mma_done, 1);
     fence_mbar_init();
@@ -111,11 +131,19 @@ __global__ void __launch_bounds__(192, 1)
     prefetch_tmap(&tm_c);
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(tmem_slot, 512);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, 512);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync_all();  // barriers of both CTAs initialised before any remote use
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -123,16 +151,20 @@ __global__ void __launch_bounds__(192, 1)
   const int M = p.m_is_R ? R : p.M;
   const int K = p.k_is_R ? R : p.K;
   GemmSchedule sch;
-  sch.init(M, p.N, K, gridDim.x, p.max_ksplit);
+  sch.init(M, p.N, K, C::kTileRows, n_workers, p.max_ksplit);
 
   if (warp == 0) {
     if (lane == 0) {
       uint32_t stage = 0, phase = 0;
       bool ok = true, any = false;
-      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x) {
+      // a pair counts both CTAs' bytes on the leader's full barriers
+      const uint32_t full_leader = PAIR ? mapa_shared(smem_u32(full), 0u) : smem_u32(full);
+      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
-        const int m0 = mt * kRowTile, n0 = nt * kBN;
+        // this CTA's 128 rows of A and (pair) its half of B's columns
+        const int m0 = mt * C::kTileRows + (int)rank * kRowTile;
+        const int n0 = nt * kBN + (int)rank * (kBN - C::kBCols);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, status, lim)) {
             ok = false;
@@ -141,18 +173,29 @@ __global__ void __launch_bounds__(192, 1)
           uint8_t* sa = stage_base + stage * kStageBytes;
           uint8_t* sb = sa + kABytes;
           const int k0 = kb * kKBlock;
-          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          if (!PAIR) {
+            mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          } else if (rank == 0) {
+            mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
+          }
+          const uint32_t fb = full_leader + stage * 8u;
+          auto load = [&](void* dst, const CUtensorMap* m, int32_t c0, int32_t c1) {
+            if (PAIR)
+              tma_load_2d_pair(dst, m, fb, c0, c1);
+            else
+              tma_load_2d(dst, m, &full[stage], c0, c1);
+          };
           if (A_MN) {
-            tma_load_2d(sa, &tm_a, &full[stage], m0, k0);
-            tma_load_2d(sa + 8192, &tm_a, &full[stage], m0 + 64, k0);
+            load(sa, &tm_a, m0, k0);
+            load(sa + 8192, &tm_a, m0 + 64, k0);
           } else {
-            tma_load_2d(sa, &tm_a, &full[stage], k0, m0);
+            load(sa, &tm_a, k0, m0);
           }
           if (B_MN) {
 #pragma unroll
-            for (int i = 0; i < kBN / 64; ++i) tma_load_2d(sb + 8192 * i, &tm_b, &full[stage], n0 + 64 * i, k0);
+            for (int i = 0; i < C::kBCols / 64; ++i) load(sb + 8192 * i, &tm_b, n0 + 64 * i, k0);
           } else {
-            tma_load_2d(sb, &tm_b, &full[stage], k0, n0);
+            load(sb, &tm_b, k0, n0);
           }
           any = true;
           if (++stage == (uint32_t)kStages) {
@@ -161,7 +204,9 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
-      if (!ok && any) {
+      if (!ok && any && rank == 0) {
+        // let every copy already issued land before the CTA can exit (in a pair,
+        // the leader's barriers also count the peer's copies)
         for (int s = 0; s < kStages; ++s) {
           const uint32_t par = ((uint32_t)s < stage) ? phase : (phase ^ 1u);
           mbar_wait_drain(&full[s], par, lim);
@@ -169,12 +214,12 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kRowTile, kBN, A_MN, B_MN);
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(C::kTileRows, kBN, A_MN, B_MN);
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < sch.n_units; u += gridDim.x, ++lt) {
+      for (int u = worker; ok && u < sch.n_units; u += n_workers, ++lt) {
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
         const int buf = lt & 1;
@@ -199,17 +244,32 @@ __global__ void __launch_bounds__(192, 1)
             // MN-major: it starts 16 rows (2048 bytes) further down; 64-wide MN blocks are 8 KB apart.
             const uint64_t ad = A_MN ? sdesc_sw128(sa + k * 2048, 8192, 1024) : sdesc_sw128(sa + k * 32, 16, 1024);
             const uint64_t bd = B_MN ? sdesc_sw128(sb + k * 2048, 8192, 1024) : sdesc_sw128(sb + k * 32, 16, 1024);
-            umma_bf16(d_tmem, ad, bd, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
+            if (PAIR)
+              umma_bf16_pair(d_tmem, ad, bd, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
+            else
+              umma_bf16(d_tmem, ad, bd, idesc, (kb != kb0 || k != 0) ? 1u : 0u);
           }
-          umma_commit(&empty[stage]);
+          if (PAIR)
+            umma_commit_pair_mc(&empty[stage], 0x3);
+          else
+            umma_commit(&empty[stage]);
           if (++stage == (uint32_t)kStages) {
             stage = 0;
             phase ^= 1u;
           }
         }
-        if (ok) umma_commit(&acc_full[buf]);
+        if (ok) {
+          if (PAIR)
+            umma_commit_pair_mc(&acc_full[buf], 0x3);
+          else
+            umma_commit(&acc_full[buf]);
+        }
       }
-      umma_commit(mma_done);
+      // every MMA issued by this thread completes before TMEM is released
+      if (PAIR)
+        umma_commit_pair_mc(mma_done, 0x1);
+      else
+        umma_commit(mma_done);
       mbar_wait_drain(mma_done, 0, lim);
     }
   } else {
@@ -218,7 +278,9 @@ __global__ void __launch_bounds__(192, 1)
     uint8_t* stg = staging + q * kStagingPerWarp;
     int lt = 0;
     int nchunk = 0;
-    for (int u = blockIdx.x; u < sch.n_units; u += gridDim.x, ++lt) {
+    // the MMA issuer (in the pair's leader) waits for every epilogue warp of the pair
+    const uint32_t acc_empty_leader = PAIR ? mapa_shared(smem_u32(acc_empty), 0u) : smem_u32(acc_empty);
+    for (int u = worker; u < sch.n_units; u += n_workers, ++lt) {
       int mt, nt, kb0, kb1;
       sch.unit(u, mt, nt, kb0, kb1);
       const int buf = lt & 1;
@@ -227,8 +289,9 @@ __global__ void __launch_bounds__(192, 1)
       if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[buf], acc_par, status, lim))) break;
       tc_fence_after();
       const bool empty_k = kb1 <= kb0;
-      const int m0 = mt * kRowTile + q * 32, n0 = nt * kBN;
-      if (!(empty_k && p.reduce)) {
+      const int m0 = mt * C::kTileRows + (int)rank * kRowTile + q * 32, n0 = nt * kBN;
+      // rows of the last tile past M (a pair's odd CTA can hold none) are not stored
+      if (!(empty_k && p.reduce) && m0 < M) {
 #pragma unroll 1
         for (int c = 0; c < kBN / 32; ++c) {
           if (n0 + c * 32 >= p.N) break;
@@ -261,37 +324,79 @@ __global__ void __launch_bounds__(192, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      if (lane == 0) {
+        if (PAIR)
+          mbar_arrive_cluster(acc_empty_leader + (uint32_t)buf * 8u);
+        else
+          mbar_arrive(&acc_empty[buf]);
+      }
     }
     if (lane == 0) bulk_wait_all<0>();
   }
 
   tc_fence_before();
-  __syncthreads();
+  if (PAIR)
+    cluster_sync_all();  // the pair's MMAs and both epilogues are done with TMEM
+  else
+    __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
+    if (PAIR)
+      tmem_dealloc_pair(tmem_base, 512);
+    else
+      tmem_dealloc(tmem_base, 512);
   }
 }
 
-template <bool A_MN, bool B_MN>
+template <bool A_MN, bool B_MN, bool PAIR>
 cudaError_t launch_impl(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c, const GemmParams& p,
                         int grid, cudaStream_t s) {
-  auto kern = k_umma_gemm<A_MN, B_MN>;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+  constexpr size_t smem = GemmCfg<PAIR>::kSmem;
+  auto kern = k_umma_gemm<A_MN, B_MN, PAIR>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, 192, kSmem, s>>>(a, b, c, p);
+  if (!PAIR) {
+    kern<<<grid, 192, smem, s>>>(a, b, c, p);
+    return cudaGetLastError();
+  }
+  // one CTA pair per two SMs, no more pairs than can be resident at once
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(192, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.gridDim = dim3((unsigned)(grid & ~1), 1, 1);
+  int max_clusters = 0;
+  e = cudaOccupancyMaxActiveClusters(&max_clusters, kern, &cfg);
+  if (e != cudaSuccess) return e;
+  if (max_clusters < 1) return cudaErrorInvalidConfiguration;
+  const int pairs = (grid / 2) < max_clusters ? (grid / 2) : max_clusters;
+  cfg.gridDim = dim3((unsigned)(2 * pairs), 1, 1);
+  e = cudaLaunchKernelEx(&cfg, kern, a, b, c, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 }  // namespace
 
+// The pair tiling stages B as 64-column MN-major boxes only: a K-major B would need
+// a 128-row tensor-map box, which the maps of this library do not provide.
 cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                         const GemmParams& p, int grid, cudaStream_t s) {
-  if (!a_mn && !b_mn) return launch_impl<false, false>(a, b, c, p, grid, s);
-  if (!a_mn && b_mn) return launch_impl<false, true>(a, b, c, p, grid, s);
-  if (a_mn && !b_mn) return launch_impl<true, false>(a, b, c, p, grid, s);
-  return launch_impl<true, true>(a, b, c, p, grid, s);
+  if (p.pair) {
+    if (!b_mn) return cudaErrorInvalidValue;
+    return a_mn ? launch_impl<true, true, true>(a, b, c, p, grid, s) : launch_impl<false, true, true>(a, b, c, p, grid, s);
+  }
+  if (!a_mn && !b_mn) return launch_impl<false, false, false>(a, b, c, p, grid, s);
+  if (!a_mn && b_mn) return launch_impl<false, true, false>(a, b, c, p, grid, s);
+  if (a_mn && !b_mn) return launch_impl<true, false, false>(a, b, c, p, grid, s);
+  return launch_impl<true, true, false>(a, b, c, p, grid, s);
 }
 
 }  // namespace opd

@@ -49,6 +49,7 @@ struct GemmParams {
   int32_t m_is_R, k_is_R;
   int32_t max_ksplit;   // 1 = whole K per tile
   int32_t reduce;       // 1 = TMA reduce-add into C, 0 = TMA store
+  int32_t pair;         // 1 = 256 x 256 tiles on CTA pairs (B must be MN-major), 0 = 128 x 256 on one CTA
   uint64_t wait_limit_ns;
 };
 

@@ -103,27 +103,30 @@ def _small_bf16(**kw):
     return synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
 
 
-@pytest.fixture(params=["bn256", "pair256"])
-def fused_bn(request, monkeypatch):
-    """Every tiling of the fused kernels: 128 x 256 tiles on one CTA, 256 x 256 tiles on a CTA pair
-    (the library reads the override on every call)."""
-    monkeypatch.setenv("OPD_KL_FUSED", request.param)
+@pytest.fixture(params=["bn256/cta1", "pair256/cta1", "pair256/pair"])
+def tiling(request, monkeypatch):
+    """Tilings of the fused kernels (128 x 256 tiles on one CTA, 256 x 256 on a CTA pair) and of the
+    gradient GEMMs (128 x 256 on one CTA, 256 x 256 on a pair); the library reads both overrides on
+    every call."""
+    fused, gemm = request.param.split("/")
+    monkeypatch.setenv("OPD_KL_FUSED", fused)
+    monkeypatch.setenv("OPD_KL_GEMM", gemm)
     return request.param
 
 
-def test_bf16_several_tiles_ragged_vocab(lib, oracle_mod, fused_bn):
+def test_bf16_several_tiles_ragged_vocab(lib, oracle_mod, tiling):
     # 3+ row tiles with a ragged last tile, several vocabulary tiles with a ragged tail,
     # K blocks 4 (student) and 6 (teacher)
     _full_check(lib, oracle_mod, _small_bf16())
 
 
-def test_bf16_ragged_hidden_sizes_and_vocab(lib, oracle_mod, fused_bn):
+def test_bf16_ragged_hidden_sizes_and_vocab(lib, oracle_mod, tiling):
     # d not a multiple of the 64-wide K block, d_s not a multiple of the 256-wide GEMM tile,
     # V not a multiple of 8 (dz pitch padding)
     _full_check(lib, oracle_mod, _small_bf16(T=300, d_s=200, d_t=136, V=1237, tau=1.3, n_traj=3, seed=12))
 
 
-def test_bf16_many_vocab_splits(lib, oracle_mod, fused_bn):
+def test_bf16_many_vocab_splits(lib, oracle_mod, tiling):
     # few row tiles and a long vocabulary: the forward splits V across many CTAs
     _full_check(lib, oracle_mod, _small_bf16(T=256, d_s=64, d_t=64, V=40000, tau=1.0, n_traj=2, traj_len=128,
                                              seed=23))
@@ -173,7 +176,7 @@ def test_all_rows_masked(lib):
 
 
 @pytest.mark.parametrize("rows", [[0], [199], [5, 6, 7, 127, 128, 129]])
-def test_few_supervised_rows(lib, oracle_mod, rows, fused_bn):
+def test_few_supervised_rows(lib, oracle_mod, rows, tiling):
     w = _small_bf16(T=200, seed=17)
     mask = np.zeros(w.T, np.uint8)
     mask[rows] = 1

@@ -36,9 +36,12 @@ def lib():
     return opd_kl
 
 
-@pytest.fixture(params=["bn256", "pair256"])
+@pytest.fixture(params=["bn256/cta1", "pair256/pair"])
 def tiling(request, monkeypatch):
-    monkeypatch.setenv("OPD_KL_FUSED", request.param)
+    """Single-CTA and CTA-pair tilings of the head kernels and of the gradient GEMMs."""
+    fused, gemm = request.param.split("/")
+    monkeypatch.setenv("OPD_KL_FUSED", fused)
+    monkeypatch.setenv("OPD_KL_GEMM", gemm)
     return request.param
 
 
