@@ -46,6 +46,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 KERNEL_SOURCES = {
     "fused_logits_fwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
     "fused_logits_bwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+    "head_logits_fwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
+    "head_logits_bwd": ["paper_2609_36608_gb300/csrc/opd_fused.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
     "gemm_dH": ["paper_2609_36608_gb300/csrc/opd_gemm.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
     "gemm_dW": ["paper_2609_36608_gb300/csrc/opd_gemm.cu", "paper_2609_36608_gb300/csrc/opd_device.cuh"],
 }
@@ -179,9 +181,11 @@ def source_hash(name):
     return h.hexdigest()
 
 
-def recorded_traffic(name, workload):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel source still matches."""
-    path = os.path.join(ROOT, "profiles", f"{name}_{workload}.txt")
+def recorded_traffic(name, workload, step_path="kl"):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source still matches
+    (profiles/<kernel>_<workload>.txt for the KL step, <kernel>_<path>_<workload>.txt otherwise)."""
+    tag = workload if step_path == "kl" else f"{step_path}_{workload}"
+    path = os.path.join(ROOT, "profiles", f"{name}_{tag}.txt")
     if not os.path.exists(path):
         return None
     text = open(path).read()
@@ -466,7 +470,7 @@ def run_gpu(args):
         per_launch = path_kernel_flops(args.path, dom, w, R)
         achieved = per_launch / (kernels[dom]["ms_per_launch"] / 1000.0) / 1e12
         peak = peaks["bf16_tflops_sustained"]
-        traffic = recorded_traffic(dom, w.name) if args.path == "kl" else None
+        traffic = recorded_traffic(dom, w.name, args.path)
         roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak, "traffic": traffic,
                     "peak_source": f"bf16_tflops_sustained of {peak_src}",

@@ -304,7 +304,7 @@ FusedParams fused_params(const Call& c) {
   fp.d_s = (int32_t)c.p.d_s;
   fp.d_t = (int32_t)c.p.d_t;
   fp.T_pad = (int32_t)c.L.T_pad;
-  fp.group_rows = env_int("OPD_KL_GROUP_ROWS", 8);
+  fp.group_rows = env_int("OPD_KL_GROUP_ROWS", 10);
   fp.k2 = (float)(1.4426950408889634 / (double)c.p.temperature);
   fp.inv_tau = 1.0f / c.p.temperature;
   fp.wait_limit_ns = kDefaultWaitLimitNs;

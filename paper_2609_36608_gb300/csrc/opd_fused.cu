@@ -69,12 +69,18 @@ struct FusedCfg {
 struct FusedSchedule {
   int n_rt, n_vt, n_vs, G, n_units;
 
-  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split, bool bwd) {
+  // Both passes walk the same units; only the forward keeps per-split statistics.
+  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split) {
     n_rt = (R + tile_rows - 1) / tile_rows;
     n_vt = (V + kBN - 1) / kBN;
+    // groups of at most G_ row tiles, as equal in size as possible
     G = G_ < 1 ? 1 : G_;
-    if (bwd || n_rt == 0) {
-      n_vs = bwd ? n_vt : 1;
+    if (n_rt > 0) {
+      const int n_groups = (n_rt + G - 1) / G;
+      G = (n_rt + n_groups - 1) / n_groups;
+    }
+    if (n_rt == 0) {
+      n_vs = 1;
     } else {
       // fewest tiles on the busiest worker, then the fewest splits
       long best = -1;
@@ -338,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int R = p.ctrl->R;
   FusedSchedule sch;
-  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit, BWD);
+  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit);
   if (!BWD && blockIdx.x == 0 && threadIdx.x == 0) p.ctrl->n_vsplit = sch.n_vs;
   const int nks = (p.d_s + kKBlock - 1) / kKBlock;
   const int nkt = (p.d_t + kKBlock - 1) / kKBlock;

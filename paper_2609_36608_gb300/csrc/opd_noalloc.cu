@@ -144,7 +144,7 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.d_s = (int32_t)p.d_s;
   fp.d_t = (int32_t)p.d_t;
   fp.T_pad = T_pad;
-  fp.group_rows = 8;
+  fp.group_rows = 10;
   fp.k2 = (float)(1.4426950408889634 / (double)p.temperature);
   fp.inv_tau = 1.0f / p.temperature;
   fp.wait_limit_ns = 2000000000ull;
