@@ -360,6 +360,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s
   gh.max_ksplit = env_int("OPD_KL_MAX_KSPLIT", kMaxKSplit);
   gh.reduce = 1;
   gh.pair = gemm_pair_mode();
+  gh.work_slot = 2;
   gh.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dH", c.s, [&] { return launch_gemm(false, true, m.dz_a_k, m.ws_b_mn, m.dhg, gh, c.dev.sm_count, c.s); }));
 
@@ -373,6 +374,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s
   gw.max_ksplit = 1;
   gw.reduce = accumulate_dW ? 1 : 0;
   gw.pair = gemm_pair_mode();
+  gw.work_slot = 3;
   gw.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dW", c.s, [&] { return launch_gemm(true, true, m.dz_a_mn, m.hsg_b_mn, m.dw, gw, c.dev.sm_count, c.s); }));
 

@@ -23,7 +23,7 @@ struct Ctrl {
   int32_t R;          // supervised rows (written by the compaction kernel)
   uint32_t status;    // kDev* bits, cleared at the start of every call
   int32_t n_vsplit;   // vocabulary splits the forward used (written by the fused forward)
-  int32_t work[4];    // work-unit counters of the fused kernels (forward, backward), zeroed per call
+  int32_t work[4];    // work-unit counters: fused forward, fused backward, dH_s GEMM, dW_s GEMM; zeroed per call
   int32_t pad[57];
 };
 

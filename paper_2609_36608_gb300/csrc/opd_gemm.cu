@@ -16,6 +16,8 @@
 // stages its own 128 rows of A and 128 of the 256 columns of B, holds its 128 x 256
 // accumulator in its own TMEM and stores it; the even CTA issues the MMAs. Per
 // byte staged from L2 this does 1.5 times the MMA work of the single-CTA tile.
+// Pairs take tiles in increasing order from a global counter (single CTAs walk a
+// fixed stride), so the pairs that read the same A rows run them at the same time.
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
@@ -34,7 +36,7 @@ struct GemmCfg {
   static constexpr uint32_t kABytes = kRowTile * kKBlock * 2;       // 16 KB
   static constexpr uint32_t kBBytes = kBCols * kKBlock * 2;         // 32 KB (16 KB in a pair)
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
-  static constexpr size_t kFixed = 1024 + 4 * kStagingPerWarp + 256;
+  static constexpr size_t kFixed = 1024 + 4 * kStagingPerWarp + 512;
   static constexpr int kStages = (int)((232448 - kFixed) / kStageBytes) > 6 ? 6 : (int)((232448 - kFixed) / kStageBytes);
   static constexpr size_t kSmem = kFixed + (size_t)kStages * kStageBytes;
   static_assert(kStages >= 4, "pipeline depth");
@@ -103,7 +105,10 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* acc_full = empty + kStages;
   uint64_t* acc_empty = acc_full + 2;
   uint64_t* mma_done = acc_empty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint64_t* unit_full = mma_done + 1;  // [kUnitRing] (pairs)
+  uint64_t* unit_empty = unit_full + kUnitRing;
+  int32_t* units = reinterpret_cast<int32_t*>(unit_empty + kUnitRing);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(units + kUnitRing);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -112,6 +117,7 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t rank = PAIR ? cluster_ctarank() : 0u;  // CTA rank within the pair
   const int worker = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
   const int n_workers = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  int32_t* counter = &p.ctrl->work[p.work_slot];
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -123,6 +129,12 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&acc_empty[b], PAIR ? 8 : 4);  // epilogue warps of the pair
     }
     mbar_init(mma_done, 1);
+    // readers of each unit slot: MMA issuer and epilogue warps of the even CTA, producer
+    // and epilogue warps of the odd one
+    for (int i = 0; i < kUnitRing; ++i) {
+      mbar_init(&unit_full[i], 1);
+      mbar_init(&unit_empty[i], 2 * 5);
+    }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -159,7 +171,25 @@ __global__ void __launch_bounds__(192, 1)
       bool ok = true, any = false;
       // a pair counts both CTAs' bytes on the leader's full barriers
       const uint32_t full_leader = PAIR ? mapa_shared(smem_u32(full), 0u) : smem_u32(full);
-      for (int u = worker; ok && u < sch.n_units; u += n_workers) {
+      int next = (PAIR && rank == 0) ? atomicAdd(counter, 1) : 0;
+      for (uint32_t k = 0; ok; ++k) {
+        int u;
+        if (!PAIR) {
+          u = worker + (int)k * n_workers;
+        } else if (rank == 0) {
+          u = next;
+          if (!publish_unit<true>(k, u, unit_full, unit_empty, units, status, lim))
+            u = -1;
+          else if (u < sch.n_units)
+            next = atomicAdd(counter, 1);  // claimed now, used by the next iteration
+        } else {
+          u = take_unit<true>(k, unit_full, unit_empty, units, true, status, lim);
+        }
+        if (u < 0) {
+          ok = false;
+          break;
+        }
+        if (u >= sch.n_units) break;
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
         // this CTA's 128 rows of A and (pair) its half of B's columns
@@ -219,7 +249,14 @@ __global__ void __launch_bounds__(192, 1)
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
-      for (int u = worker; ok && u < sch.n_units; u += n_workers, ++lt) {
+      for (uint32_t k = 0; ok; ++k, ++lt) {
+        const int u = PAIR ? take_unit<true>(k, unit_full, unit_empty, units, false, status, lim)
+                           : worker + (int)k * n_workers;
+        if (u < 0) {
+          ok = false;
+          break;
+        }
+        if (u >= sch.n_units) break;
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
         const int buf = lt & 1;
@@ -280,7 +317,10 @@ __global__ void __launch_bounds__(192, 1)
     int nchunk = 0;
     // the MMA issuer (in the pair's leader) waits for every epilogue warp of the pair
     const uint32_t acc_empty_leader = PAIR ? mapa_shared(smem_u32(acc_empty), 0u) : smem_u32(acc_empty);
-    for (int u = worker; u < sch.n_units; u += n_workers, ++lt) {
+    for (uint32_t k = 0;; ++k, ++lt) {
+      const int u = PAIR ? take_unit_warp<true>(k, unit_full, unit_empty, units, rank != 0, status, lim)
+                         : worker + (int)k * n_workers;
+      if (u < 0 || u >= sch.n_units) break;
       int mt, nt, kb0, kb1;
       sch.unit(u, mt, nt, kb0, kb1);
       const int buf = lt & 1;

@@ -50,6 +50,7 @@ struct GemmParams {
   int32_t max_ksplit;   // 1 = whole K per tile
   int32_t reduce;       // 1 = TMA reduce-add into C, 0 = TMA store
   int32_t pair;         // 1 = 256 x 256 tiles on CTA pairs (B must be MN-major), 0 = 128 x 256 on one CTA
+  int32_t work_slot;    // pairs: the Ctrl::work counter this launch takes its tiles from (2 or 3)
   uint64_t wait_limit_ns;
 };
 
