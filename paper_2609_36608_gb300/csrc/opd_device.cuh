@@ -37,6 +37,18 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// ------------------------------------------------------------------- math --
+
+// 2^x by the PTX instruction ex2.approx.ftz.f32 (the special-function unit's
+// base-2 exponential): results below 2^-126 flush to zero and 2^-inf = 0. The
+// epilogues only take it of x - max <= 0, where a flushed term is below 2^-126 of
+// the row's largest one. A single instruction, where exp2f adds range handling.
+__device__ __forceinline__ float ex2_ftz(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // ---------------------------------------------------------------- mbarrier --
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {

@@ -143,10 +143,10 @@ __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint3
   // k2 > 0, so the scaled maximum is the maximum of the scaled values
   const float nms = fmaxf(ms, cms * k2);
   const float nmt = fmaxf(mt, cmt * k2);
-  const float scs = exp2f(ms - nms);
+  const float scs = ex2_ftz(ms - nms);
   Ss *= scs;
   A *= scs;
-  St *= exp2f(mt - nmt);
+  St *= ex2_ftz(mt - nmt);
   ms = nms;
   mt = nmt;
 #pragma unroll
@@ -154,10 +154,10 @@ __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint3
     if (!PARTIAL || j < nvalid) {
       const float zs = __uint_as_float(rs[j]);
       const float zt = __uint_as_float(tv[OFF + j]);
-      const float e = exp2f(fmaf(zs, k2, -ms));
+      const float e = ex2_ftz(fmaf(zs, k2, -ms));
       Ss += e;
       A = fmaf(e, zs - zt, A);
-      St += exp2f(fmaf(zt, k2, -mt));
+      St += ex2_ftz(fmaf(zt, k2, -mt));
     }
   }
 }
@@ -190,7 +190,7 @@ __device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kCol
     for (int e = 0; e < 2; ++e) {
       const float zs = __uint_as_float(rs[2 * j + e]);
       const float zt = __uint_as_float(tv[C * 32 + 2 * j + e]);
-      const float ps = exp2f(fmaf(zs, k2, -b1));
+      const float ps = ex2_ftz(fmaf(zs, k2, -b1));
       dz2[e] = ps * fmaf(zs - zt, kc, -cc);
     }
     w[j] = pack_bf16x2(dz2[0], dz2[1]);
@@ -211,11 +211,11 @@ __device__ __forceinline__ void fold_chunk1(const uint32_t (&rs)[32], int nvalid
   for (int j = 0; j < 32; ++j)
     if (!PARTIAL || j < nvalid) cm = fmaxf(cm, __uint_as_float(rs[j]));
   const float nm = fmaxf(m, cm * k2);
-  S *= exp2f(m - nm);
+  S *= ex2_ftz(m - nm);
   m = nm;
 #pragma unroll
   for (int j = 0; j < 32; ++j)
-    if (!PARTIAL || j < nvalid) S += exp2f(fmaf(__uint_as_float(rs[j]), k2, -m));
+    if (!PARTIAL || j < nvalid) S += ex2_ftz(fmaf(__uint_as_float(rs[j]), k2, -m));
 }
 
 template <int C>
@@ -243,7 +243,7 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int col = C * 32 + 2 * j + e;
-      const float p = exp2f(fmaf(__uint_as_float(rs[2 * j + e]), k2, -b1));
+      const float p = ex2_ftz(fmaf(__uint_as_float(rs[2 * j + e]), k2, -b1));
       dz2[e] = coef * ((col == x_rel ? 1.0f : 0.0f) - p);
     }
     w[j] = pack_bf16x2(dz2[0], dz2[1]);
@@ -676,7 +676,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&merge_empty[q]);
         const float Ms = fmaxf(ms, ms1);
-        const float f0 = exp2f(ms - Ms), f1 = exp2f(ms1 - Ms);
+        const float f0 = ex2_ftz(ms - Ms), f1 = ex2_ftz(ms1 - Ms);
         Ss = Ss * f0 + Ss1 * f1;
         ms = Ms;
         const size_t plane = (size_t)p.T_pad;
@@ -686,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (HEADS == 2) {
           const float Mt = fmaxf(mt, mt1);
           A = A * f0 + A1 * f1;
-          St = St * exp2f(mt - Mt) + St1 * exp2f(mt1 - Mt);
+          St = St * ex2_ftz(mt - Mt) + St1 * ex2_ftz(mt1 - Mt);
           mt = Mt;
           base[2 * plane] = A;
           base[3 * plane] = mt;
