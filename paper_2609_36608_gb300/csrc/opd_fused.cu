@@ -125,13 +125,54 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, 
   }
 }
 
+// Maximum of the 32 values of one chunk (three-input max, 16 instructions).
+__device__ __forceinline__ float chunk_max(const uint32_t* v) {
+  float m = fmaxf(__uint_as_float(v[0]), __uint_as_float(v[1]));
+#pragma unroll
+  for (int j = 2; j < 32; j += 2) m = fmax3(m, __uint_as_float(v[j]), __uint_as_float(v[j + 1]));
+  return m;
+}
+
 // Fold 32 columns (or the first nvalid of them) of one row into the running
 // base-2 statistics: student logits in rs, teacher logits in tv[OFF..OFF+31].
 // Indices stay compile-time so the values stay in registers. x = z k2 with
-// k2 = log2(e) / tau; A is kept in raw logit units (times k2 at the end).
+// k2 = log2(e) / tau; A is kept in raw logit units (times k2 at the end). A full
+// chunk runs on paired fp32 instructions, two columns per instruction.
 template <bool PARTIAL, int OFF>
 __device__ __forceinline__ void fold_chunk(const uint32_t (&rs)[32], const uint32_t (&tv)[kColsPerWarp], int nvalid,
                                            float k2, float& ms, float& Ss, float& A, float& mt, float& St) {
+  if constexpr (!PARTIAL) {
+    const float nms = fmaxf(ms, chunk_max(rs) * k2);  // k2 > 0: max of scaled = scaled max
+    const float nmt = fmaxf(mt, chunk_max(tv + OFF) * k2);
+    const float scs = ex2_ftz(ms - nms);
+    Ss *= scs;
+    A *= scs;
+    St *= ex2_ftz(mt - nmt);
+    ms = nms;
+    mt = nmt;
+    const uint64_t k22 = f2_pack(k2, k2), nms2 = f2_pack(-ms, -ms), nmt2 = f2_pack(-mt, -mt);
+    uint64_t S2 = f2_pack(0.f, 0.f), A2 = S2, T2 = S2;
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      const uint64_t zs = f2_pack(__uint_as_float(rs[j]), __uint_as_float(rs[j + 1]));
+      const uint64_t zt = f2_pack(__uint_as_float(tv[OFF + j]), __uint_as_float(tv[OFF + j + 1]));
+      float a, b;
+      f2_unpack(f2_fma(zs, k22, nms2), a, b);
+      const uint64_t e = f2_pack(ex2_ftz(a), ex2_ftz(b));
+      S2 = f2_add(S2, e);
+      A2 = f2_fma(e, f2_sub(zs, zt), A2);
+      f2_unpack(f2_fma(zt, k22, nmt2), a, b);
+      T2 = f2_add(T2, f2_pack(ex2_ftz(a), ex2_ftz(b)));
+    }
+    float lo, hi;
+    f2_unpack(S2, lo, hi);
+    Ss += lo + hi;
+    f2_unpack(A2, lo, hi);
+    A += lo + hi;
+    f2_unpack(T2, lo, hi);
+    St += lo + hi;
+    return;
+  }
   float cms = -INFINITY, cmt = -INFINITY;
 #pragma unroll
   for (int j = 0; j < 32; ++j) {
@@ -183,6 +224,8 @@ __device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kCol
   uint32_t rs[32];
   tmem_ld32(ts + C * 32, rs);
   uint32_t w[16];
+  // scalar: with the 128 teacher registers live, paired operands cost more moves and
+  // spills than they save here (measured)
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
     float dz2[2];
@@ -206,6 +249,23 @@ __device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kCol
 // One head: 32 columns of one row folded into the running base-2 (max, sum).
 template <bool PARTIAL>
 __device__ __forceinline__ void fold_chunk1(const uint32_t (&rs)[32], int nvalid, float k2, float& m, float& S) {
+  if constexpr (!PARTIAL) {
+    const float nm = fmaxf(m, chunk_max(rs) * k2);
+    S *= ex2_ftz(m - nm);
+    m = nm;
+    const uint64_t k22 = f2_pack(k2, k2), nm2 = f2_pack(-m, -m);
+    uint64_t S2 = f2_pack(0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      float a, b;
+      f2_unpack(f2_fma(f2_pack(__uint_as_float(rs[j]), __uint_as_float(rs[j + 1])), k22, nm2), a, b);
+      S2 = f2_add(S2, f2_pack(ex2_ftz(a), ex2_ftz(b)));
+    }
+    float lo, hi;
+    f2_unpack(S2, lo, hi);
+    S += lo + hi;
+    return;
+  }
   float cm = -INFINITY;
 #pragma unroll
   for (int j = 0; j < 32; ++j)
@@ -237,16 +297,17 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
   uint32_t rs[32];
   tmem_ld32(ts + C * 32, rs);
   uint32_t w[16];
+  const uint64_t k22 = f2_pack(k2, k2), nb2 = f2_pack(-b1, -b1), coef2 = f2_pack(coef, coef);
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
-    float dz2[2];
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const int col = C * 32 + 2 * j + e;
-      const float p = ex2_ftz(fmaf(__uint_as_float(rs[2 * j + e]), k2, -b1));
-      dz2[e] = coef * ((col == x_rel ? 1.0f : 0.0f) - p);
-    }
-    w[j] = pack_bf16x2(dz2[0], dz2[1]);
+    // two columns per instruction: dz = coef (1[col = x] - p), p = 2^(z k2 - b1)
+    const int col = C * 32 + 2 * j;
+    float a, b;
+    f2_unpack(f2_fma(f2_pack(__uint_as_float(rs[2 * j]), __uint_as_float(rs[2 * j + 1])), k22, nb2), a, b);
+    const uint64_t p = f2_pack(ex2_ftz(a), ex2_ftz(b));
+    const uint64_t hot = f2_pack(col == x_rel ? 1.0f : 0.0f, col + 1 == x_rel ? 1.0f : 0.0f);
+    f2_unpack(f2_mul(coef2, f2_sub(hot, p)), a, b);
+    w[j] = pack_bf16x2(a, b);
   }
   const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
   const uint32_t jb = (uint32_t)(C & 1) * 4u;
