@@ -157,6 +157,11 @@ def max_over_ranks(x: float, world: int, device) -> float:
     return float(t.item())
 
 
+def whole_job_rate(units_per_rank_step: int, steps: int, world: int, max_ms: float) -> float:
+    """Units all ranks processed per second, over the slowest rank's time (weak scaling)."""
+    return units_per_rank_step * steps * world / (max_ms / 1000.0)
+
+
 # -------------------------------------------------------------------- flops
 
 def step_flops(w, R):
@@ -424,7 +429,7 @@ def run_gpu(args):
         raise RuntimeError("device status after the timed region is not OK")
     ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_step = ms / args.steps
-    value = R * args.steps * world / (ms / 1000.0)
+    value = whole_job_rate(R, args.steps, world, ms)
 
     # end to end through the same C ABI: the step's inputs from pinned host memory, its
     # per-token result back to the host every step
@@ -452,7 +457,7 @@ def run_gpu(args):
     torch.cuda.synchronize()
     barrier(world)
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-    e2e_value = R * args.steps * world / (e2e_ms / 1000.0)
+    e2e_value = whole_job_rate(R, args.steps, world, e2e_ms)
 
     if rank != 0:
         torch.distributed.destroy_process_group() if world > 1 else None
