@@ -352,7 +352,8 @@ def path_kernel_flops(path, name, w, R):
 
 
 def path_cpu_baseline(path, w, lay, x, args):
-    """The oracle, as it stands, on a bounded row sample of the same workload."""
+    """The oracle, as it stands, on a bounded row sample of the same workload: on every host
+    core, and on one core for a smaller sample."""
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
@@ -360,24 +361,39 @@ def path_cpu_baseline(path, w, lay, x, args):
     if path == "kl":
         host = host_inputs(x)
         g = np.where(lay.mask != 0, opd_seq_weights(lay), 0.0)
-        rate, dt = oracle_rate(w, host, lay, g, rows, threads)
+
+        def run(rs, n):
+            oracle.opd_kl(host["H_s"], host["H_t"], host["W_s"], host["W_t"], lay.mask, g, w.tau, rows=rs,
+                          want_dH=True, want_dW=True, n_threads=n)
         what = "float64 logits, KL, dH_s rows and their dW_s contribution"
     else:
         tokens = synth.token_ids(w.seed, w.T, w.V)
-        t0 = time.perf_counter()
         if path == "score":
-            oracle.score(synth.host_values(x["H_t"]), synth.host_values(x["W_t"]), tokens, w.tau, rows=rows,
-                         n_threads=threads)
+            H, W = synth.host_values(x["H_t"]), synth.host_values(x["W_t"])
+
+            def run(rs, n):
+                oracle.score(H, W, tokens, w.tau, rows=rs, n_threads=n)
             what = "float64 teacher log-partition and token log-probabilities"
         else:
-            T = w.T
-            oracle.surrogate(synth.host_values(x["H_s"]), synth.host_values(x["W_s"]), tokens, np.full(T, -7.0),
-                             np.full(T, -7.0), lay.mask, np.ones(T), w.tau, rows=rows, n_threads=threads)
+            H, W, T = synth.host_values(x["H_s"]), synth.host_values(x["W_s"]), w.T
+
+            def run(rs, n):
+                oracle.surrogate(H, W, tokens, np.full(T, -7.0), np.full(T, -7.0), lay.mask, np.ones(T), w.tau,
+                                 rows=rs, n_threads=n)
             what = "float64 student logits, dual-clip loss, dH_s rows and their dW_s contribution"
-        dt = time.perf_counter() - t0
-        rate = len(rows) / dt
-    return {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"{len(rows)} supervised rows of {w.name}: {what} ({dt:.1f} s)"}
+
+    def timed(rs, n):
+        t0 = time.perf_counter()
+        run(rs, n)
+        return time.perf_counter() - t0
+
+    dt = timed(rows, threads)
+    rows1 = rows[:max(1, min(len(rows), args.cpu_rows_1t))]
+    dt1 = timed(rows1, 1)
+    return {"value": len(rows) / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{len(rows)} supervised rows of {w.name}: {what} ({dt:.1f} s)",
+            "value_1_thread": len(rows1) / dt1,
+            "sample_1_thread": f"the first {len(rows1)} of those rows on one core ({dt1:.1f} s)"}
 
 
 def opd_seq_weights(lay):
@@ -577,6 +593,7 @@ def main():
                     help="kl: the reverse-KL step (default, the headline); surrogate: the sampled-token "
                          "dual-clip surrogate; score: teacher token scoring")
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
+    ap.add_argument("--cpu-rows-1t", type=int, default=4, help="rows of the one-core CPU-oracle sample")
     ap.add_argument("--ref-rows", type=int, default=8, help="rows per step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--calibrate", type=float, default=0.0, metavar="SECONDS",
