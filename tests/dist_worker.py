@@ -21,7 +21,9 @@ def main():
     slowest = bench.max_over_ranks(ms, world, "cpu")
     rate = bench.whole_job_rate(1000, 5, world, slowest)
     bench.barrier(world)
-    print(json.dumps({"rank": rank, "world": world, "max_ms": slowest, "rate": rate}), flush=True)
+    # one file per rank: the ranks' standard outputs interleave under torch.distributed.run
+    with open(os.path.join(os.environ["OPD_TEST_OUT"], f"rank{rank}.json"), "w") as f:
+        json.dump({"rank": rank, "world": world, "max_ms": slowest, "rate": rate}, f)
     torch.distributed.destroy_process_group()
 
 

@@ -183,6 +183,23 @@ def test_few_supervised_rows(lib, oracle_mod, rows, tiling):
     _full_check(lib, oracle_mod, w, mask=mask)
 
 
+@pytest.mark.parametrize("shape", [
+    dict(T=40, d_s=8, d_t=16, V=2),     # two-token vocabulary, hidden sizes far below one K block
+    dict(T=100, d_s=16, d_t=8, V=64),   # the whole vocabulary inside a quarter of one tile
+    dict(T=1, d_s=64, d_t=128, V=300),  # a single token
+])
+def test_shapes_below_one_tile(lib, oracle_mod, shape, tiling):
+    w = _small_bf16(n_traj=1, traj_len=shape["T"], seed=21, **shape)
+    mask = (np.arange(w.T) % 3 != 1).astype(np.uint8)
+    mask[0] = 1
+    _full_check(lib, oracle_mod, w, mask=mask)
+
+
+def test_fp32_two_token_vocabulary(lib, oracle_mod):
+    w = synth.scaled(synth.WORKLOADS["tiny_fp32"], V=2, d_s=8, d_t=16, seed=22)
+    _full_check(lib, oracle_mod, w, tight=True)
+
+
 def test_student_equals_teacher_gives_zero(lib):
     w = _small_bf16(T=256, d_t=256, seed=18)
     lay = synth.layout(w)

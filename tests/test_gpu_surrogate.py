@@ -136,6 +136,31 @@ def test_surrogate_small(lib, oracle_mod, tiling):
     assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
 
 
+@pytest.mark.parametrize("shape", [dict(T=50, d_s=8, V=2), dict(T=90, d_s=16, V=64)])
+def test_surrogate_and_scoring_below_one_tile(lib, oracle_mod, shape, tiling):
+    w = _case(n_traj=1, traj_len=shape["T"], seed=33, **shape)
+    mask = (np.arange(w.T) % 4 != 2).astype(np.uint8)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    lse, lp = _score(lib, w, x["H_s"], x["W_s"], tokens, mask)
+    sup = mask != 0
+    ref_lse, ref_lp = oracle_mod.score(Hs, Ws, tokens, w.tau, rows=np.flatnonzero(sup))
+    _close(lse[sup], ref_lse, 1e-4, 1e-4, "lse")
+    _close(lp[sup], ref_lp, 1e-4, 1e-4, "logp")
+    _, lp_full = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = (lp_full - _clear_offsets(4, w.T)).astype(np.float32)
+    adv = np.random.default_rng(5).choice([-1.0, 1.0], w.T) * np.random.default_rng(6).uniform(0.2, 1.5, w.T)
+    logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
+    weights = np.where(sup, 1.0 / max(int(sup.sum()), 1), 0.0).astype(np.float32)
+    loss, lp2, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, mask, weights)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               mask, weights.astype(np.float64), w.tau)
+    _close(loss, ref.loss, 1e-4, 2e-3, "loss")
+    assert _rel(dH, ref.dH_s) <= 1e-2, _rel(dH, ref.dH_s)
+    assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
+
+
 def test_surrogate_on_policy_and_accumulate(lib, oracle_mod):
     # rho = 1: the surrogate's gradient is the policy gradient -A (1[k = x] - p) / tau
     w = _case(T=300, d_s=128, V=2048, tau=1.0, n_traj=3, seed=33)

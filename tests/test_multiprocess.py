@@ -20,17 +20,17 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def _torchrun(args, timeout=600):
+def _torchrun(args, timeout=600, env_extra=None):
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
            "--master-addr", "127.0.0.1", "--master-port", str(_free_port())] + args
-    env = dict(os.environ, OMP_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    env = dict(os.environ, OMP_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="", **(env_extra or {}))
     return subprocess.run(cmd, capture_output=True, text=True, timeout=timeout, cwd=ROOT, env=env)
 
 
-def test_two_gloo_ranks_agree_on_the_slowest_time_and_the_job_rate():
-    out = _torchrun([os.path.join(ROOT, "tests", "dist_worker.py")])
+def test_two_gloo_ranks_agree_on_the_slowest_time_and_the_job_rate(tmp_path):
+    out = _torchrun([os.path.join(ROOT, "tests", "dist_worker.py")], env_extra={"OPD_TEST_OUT": str(tmp_path)})
     assert out.returncode == 0, out.stderr[-3000:]
-    lines = [json.loads(l) for l in out.stdout.splitlines() if l.startswith("{")]
+    lines = [json.loads((tmp_path / f"rank{r}.json").read_text()) for r in range(2)]
     assert sorted(d["rank"] for d in lines) == [0, 1]
     for d in lines:
         assert d["world"] == 2
