@@ -41,6 +41,15 @@
  * opd_kl_get_status. Nothing ever traps the GPU.
  *
  * Streams are passed as void* and are cudaStream_t values (NULL = legacy default stream).
+ * No call synchronises the host, so a sequence of calls can be captured in a CUDA graph.
+ *
+ * Tuning overrides, read from the environment at every call (defaults are the
+ * measured best on GB300):
+ *   OPD_KL_FUSED=bn256|pair256  fused-kernel tiling: 128 x 256 tiles on one CTA, or
+ *                               256 x 256 tiles on a CTA pair (default)
+ *   OPD_KL_GEMM=cta1|pair       gradient-GEMM tiling, same two choices (default pair)
+ *   OPD_KL_GROUP_ROWS=n         row tiles walked together in L2 (default 10)
+ *   OPD_KL_MAX_KSPLIT=n         largest K split of the dH_s GEMM (default 16)
  */
 #ifndef OPD_KL_H
 #define OPD_KL_H
