@@ -15,7 +15,7 @@
 // Roles: warp 0 issues TMA loads, warp 1 allocates TMEM and issues the MMAs from
 // one thread, eight epilogue warps drain TMEM (TMEM lane = tile row; the two
 // warps of each lane quadrant take 128 columns each). Persistent: work units (row
-// tile, vocabulary range) are walked grid-strided.
+// tile, vocabulary range) are taken in order from a global counter.
 //
 // TMEM holds one tile: teacher accumulator in columns [0,256), student in
 // [256,512). Each tile computes the teacher segment first and signals it on its
@@ -29,7 +29,8 @@
 // 256 rows per tile, 128 in each CTA's TMEM; each CTA stages its own 128 rows of
 // H and 128 of the 256 rows of W, the even-ranked CTA issues the MMAs, and both
 // CTAs' TMA completions are counted on the leader's barriers. Per byte staged
-// from L2 this does twice the MMA work of a single-CTA 128 x 256 tile.
+// from L2 this does 1.5 times the MMA work of a single-CTA 128 x 256 tile (each
+// CTA stages half of W's rows).
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
