@@ -83,12 +83,17 @@ struct FusedSchedule {
     if (n_rt == 0) {
       n_vs = 1;
     } else {
-      // fewest tiles on the busiest worker, then the fewest splits
+      // fewest tiles on the busiest worker, then the fewest splits; at least enough
+      // splits that the units running at once span one raster group of row tiles, so
+      // the group's hidden-state tiles stay in L2 (with fewer splits every worker
+      // streams the whole vocabulary against its own row tile and H leaves L2)
       long best = -1;
-      n_vs = 1;
       const int cap = max_split < 1 ? 1 : (max_split > kMaxVSplit ? kMaxVSplit : max_split);
       const int max_vs = n_vt < cap ? n_vt : cap;
-      for (int s = 1; s <= max_vs; ++s) {
+      int min_vs = (workers + G - 1) / G;
+      min_vs = min_vs < 1 ? 1 : (min_vs > max_vs ? max_vs : min_vs);
+      n_vs = min_vs;
+      for (int s = min_vs; s <= max_vs; ++s) {
         const long waves = ((long)n_rt * s + workers - 1) / workers;
         const long cost = waves * ((n_vt + s - 1) / s);
         if (best < 0 || cost < best) {
