@@ -32,7 +32,8 @@
  * including the workspace; the library allocates nothing, keeps no pointer
  * after a call returns, and enqueues all work on the given stream without
  * synchronising it (unless OPD_KL_SYNC_CHECK=1 is set in the environment, which
- * makes every call synchronise and report device-side errors).
+ * makes every call scan its float outputs for NaN and infinity, synchronise, and
+ * report device-side errors, OPD_ERR_NONFINITE included).
  *
  * Errors: every argument is validated on the host before any launch; a bad
  * argument returns OPD_ERR_INVALID_ARG or OPD_ERR_UNSUPPORTED and launches
@@ -67,7 +68,8 @@ typedef enum {
   OPD_ERR_UNSUPPORTED = 2, /* valid but not handled (e.g. bf16 with d % 8 != 0) */
   OPD_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed */
   OPD_ERR_TIMEOUT = 4,     /* a device-side bounded wait ran out (see opd_kl_get_status) */
-  OPD_ERR_NONFINITE = 5    /* reserved: non-finite inputs are undefined behaviour, not checked */
+  OPD_ERR_NONFINITE = 5    /* debug mode (OPD_KL_SYNC_CHECK=1) only: an output holds NaN or infinity.
+                              Inputs must be finite; outside debug mode nothing is checked */
 } opd_status;
 
 typedef enum { OPD_DTYPE_BF16 = 0, OPD_DTYPE_F32 = 1 } opd_dtype;

@@ -226,9 +226,27 @@ opd_status begin_call(Call& c, const opd_problem* problem, void* workspace, size
   return OPD_OK;
 }
 
-opd_status finish_call(const Call& c) {
+// Output buffers a call wrote (pointer, element count), checked for non-finite
+// values in debug mode.
+struct Outputs {
+  const float* p[5] = {};
+  size_t n[5] = {};
+  int k = 0;
+  Outputs& add(const float* q, size_t m) {
+    if (q && m && k < 5) {
+      p[k] = q;
+      n[k++] = m;
+    }
+    return *this;
+  }
+};
+
+opd_status finish_call(const Call& c, const Outputs& out = Outputs()) {
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
-  if (env_flag("OPD_KL_SYNC_CHECK")) return opd_kl_get_status(c.ws, c.L.total, c.s);
+  if (env_flag("OPD_KL_SYNC_CHECK")) {
+    for (int i = 0; i < out.k; ++i) OPD_CUDA(launch_check_finite(out.p[i], out.n[i], c.ctrl(), c.dev.sm_count, c.s));
+    return opd_kl_get_status(c.ws, c.L.total, c.s);
+  }
   return OPD_OK;
 }
 
@@ -398,6 +416,10 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
     if (!aligned(dW_s, a) || !aligned(dH_s, a)) return OPD_ERR_INVALID_ARG;
   }
   const float* stats = do_fwd ? stats_out : stats_in;
+  Outputs outputs;
+  const size_t Tn = (size_t)T;
+  if (do_fwd) outputs.add(kl_out, Tn).add(stats_out, 3 * Tn);
+  if (do_bwd) outputs.add(dH_s, Tn * (size_t)c.p.d_s).add(dW_s, (size_t)c.p.V * (size_t)c.p.d_s);
 
   OPD_TRY(prologue(c, H_s, H_t, mask));
   if (c.p.dtype == OPD_DTYPE_F32) {
@@ -416,14 +438,14 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
                                     (int32_t)c.p.V, c.p.temperature, c.idx(), c.pos(), c.ctrl(), stats, grad_kl,
                                     reinterpret_cast<float*>(c.ws + c.L.dz), dH_s, dW_s, accumulate_dW, c.s);
       }));
-    return finish_call(c);
+    return finish_call(c, outputs);
   }
 
   Maps m;
   OPD_TRY(encode_maps(c, W_s, W_t, dW_s, m, do_bwd));
   if (do_fwd) OPD_TRY(forward_body(c, m, kl_out, stats_out));
   if (do_bwd) OPD_TRY(backward_body(c, m, stats, grad_kl, dH_s, dW_s, accumulate_dW));
-  return finish_call(c);
+  return finish_call(c, outputs);
 }
 
 // Single-head path: compaction, gather of the head's rows, fused forward statistics,
@@ -481,7 +503,12 @@ opd_status head_call(const opd_problem* problem, const void* H, const void* W, c
                    [&] { return launch_head_backward(m.hs, m.ws, m.dz_store, fp, c.dev.sm_count, c.s); }));
     OPD_TRY(gradient_gemms(c, m, dH, dW, accumulate_dW));
   }
-  return finish_call(c);
+  Outputs outputs;
+  const size_t Tn = (size_t)T;
+  outputs.add(lse_out, Tn).add(logp_out, Tn);
+  if (surrogate)
+    outputs.add(loss_out, Tn).add(dH, Tn * (size_t)c.p.d_s).add(dW, (size_t)c.p.V * (size_t)c.p.d_s);
+  return finish_call(c, outputs);
 }
 
 }  // namespace
@@ -581,7 +608,12 @@ opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* 
                                       loss_in ? loss_out : nullptr, workspace, dev.sm_count, s);
   }));
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
-  if (env_flag("OPD_KL_SYNC_CHECK")) return opd_kl_get_status(workspace, workspace_bytes, stream);
+  if (env_flag("OPD_KL_SYNC_CHECK")) {
+    Ctrl* ctrl = static_cast<Ctrl*>(workspace);
+    OPD_CUDA(launch_check_finite(w_out, w_out ? (size_t)T : 0, ctrl, dev.sm_count, s));
+    OPD_CUDA(launch_check_finite(loss_in ? loss_out : nullptr, 1, ctrl, dev.sm_count, s));
+    return opd_kl_get_status(workspace, workspace_bytes, stream);
+  }
   return OPD_OK;
 }
 
@@ -597,6 +629,7 @@ opd_status opd_kl_get_status(void* workspace, size_t workspace_bytes, void* stre
   if (st & kDevTimeout) return OPD_ERR_TIMEOUT;
   if (st & kDevBadToken) return OPD_ERR_INVALID_ARG;
   if (st & kDevBadShape) return OPD_ERR_UNSUPPORTED;
+  if (st & kDevNonFinite) return OPD_ERR_NONFINITE;
   return OPD_OK;
 }
 

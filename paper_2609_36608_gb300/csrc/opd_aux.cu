@@ -230,6 +230,20 @@ cudaError_t launch_scatter_rows(const float* src_g, int32_t cols, const int32_t*
   return cudaGetLastError();
 }
 
+// Debug check of an output buffer: any NaN or infinity sets kDevNonFinite.
+__global__ void k_check_finite(const float* __restrict__ p, size_t n, uint32_t* status) {
+  bool bad = false;
+  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+    bad |= !isfinite(p[i]);
+  if (__any_sync(0xffffffffu, bad) && (threadIdx.x & 31) == 0) atomicOr(status, kDevNonFinite);
+}
+
+cudaError_t launch_check_finite(const float* p, size_t n, Ctrl* ctrl, int n_sm, cudaStream_t s) {
+  if (!p || n == 0) return cudaSuccess;
+  k_check_finite<<<grid_for((long)((n + 3) / 4), n_sm, 256), 256, 0, s>>>(p, n, &ctrl->status);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_selftest_timeout(Ctrl* ctrl, uint64_t limit_ns, cudaStream_t s) {
   k_selftest_timeout<<<1, 32, 0, s>>>(ctrl, limit_ns);
   return cudaGetLastError();

@@ -16,6 +16,7 @@ enum : uint32_t {
   kDevTimeout = 1u,    // a bounded wait ran out
   kDevBadShape = 2u,   // a kernel found a size it cannot handle
   kDevBadToken = 4u,   // a token id outside [0, V)
+  kDevNonFinite = 8u,  // debug check: an output holds NaN or infinity
 };
 
 // Control block at the head of the workspace.

@@ -89,6 +89,8 @@ cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t
 cudaError_t launch_scatter_rows(const float* src_g, int32_t cols, const int32_t* pos, int32_t T, float* dst,
                                 int n_sm, cudaStream_t s);
 cudaError_t launch_selftest_timeout(Ctrl* ctrl, uint64_t limit_ns, cudaStream_t s);
+// Debug mode only: sets the non-finite status bit if p[0..n) holds a NaN or infinity.
+cudaError_t launch_check_finite(const float* p, size_t n, Ctrl* ctrl, int n_sm, cudaStream_t s);
 
 // fp32 CUDA-core path (opd_simt.cu)
 cudaError_t launch_simt_forward(const float* H_s, const float* H_t, const float* W_s, const float* W_t,

@@ -156,10 +156,14 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
 
   const char* sync = std::getenv("OPD_KL_SYNC_CHECK");
   if (sync && sync[0] && sync[0] != '0') {
+    if (launch_check_finite(kl_out, (size_t)T, ctrl, sms, s) != cudaSuccess ||
+        launch_check_finite(stats, 3 * (size_t)T, ctrl, sms, s) != cudaSuccess)
+      return OPD_ERR_CUDA;
     uint32_t st = 0;
     if (cudaStreamSynchronize(s) != cudaSuccess) return OPD_ERR_CUDA;
     if (cudaMemcpy(&st, &ctrl->status, sizeof st, cudaMemcpyDeviceToHost) != cudaSuccess) return OPD_ERR_CUDA;
     if (st & kDevTimeout) return OPD_ERR_TIMEOUT;
+    if (st & kDevNonFinite) return OPD_ERR_NONFINITE;
   }
   return OPD_OK;
 }

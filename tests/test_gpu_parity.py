@@ -255,6 +255,25 @@ def test_cuda_graph_capture_and_replay(lib, oracle_mod):
     assert _rel(dW.cpu().numpy(), ref.dW_s) <= GRAD_REL
 
 
+def test_debug_mode_reports_non_finite_outputs(lib, monkeypatch):
+    """With OPD_KL_SYNC_CHECK=1 every call scans its outputs: a NaN in one supervised hidden row
+    comes back as OPD_ERR_NONFINITE. Without it nothing is checked (inputs must be finite)."""
+    w = _small_bf16(T=128, d_s=64, d_t=64, V=300, n_traj=1, traj_len=128, seed=26)
+    x = synth.hidden_and_heads(w, "cuda")
+    mask = np.ones(w.T, np.uint8)
+    monkeypatch.setenv("OPD_KL_SYNC_CHECK", "1")
+    clean = _run(lib, w, x, mask, np.ones(w.T))
+    assert np.isfinite(clean["kl"]).all()
+    x["H_s"] = x["H_s"].clone()
+    x["H_s"][5, 3] = float("nan")
+    with pytest.raises(lib.OpdError) as err:
+        _run(lib, w, x, mask, np.ones(w.T))
+    assert err.value.status == lib.OPD_ERR_NONFINITE
+    monkeypatch.delenv("OPD_KL_SYNC_CHECK")
+    out = _run(lib, w, x, mask, np.ones(w.T))
+    assert np.isnan(out["kl"][5]) and np.isfinite(np.delete(out["kl"], 5)).all()
+
+
 def test_student_equals_teacher_gives_zero(lib):
     w = _small_bf16(T=256, d_t=256, seed=18)
     lay = synth.layout(w)
