@@ -274,6 +274,37 @@ def test_debug_mode_reports_non_finite_outputs(lib, monkeypatch):
     assert np.isnan(out["kl"][5]) and np.isfinite(np.delete(out["kl"], 5)).all()
 
 
+def test_empty_batch(lib):
+    """T = 0: every call succeeds; dW_s is zeroed, or left untouched when accumulating."""
+    d_s, d_t, V = 64, 128, 300
+    prob = lib.make_problem(0, d_s, d_t, V, lib.OPD_DTYPE_BF16, 1.0)
+    ws = lib.allocate_workspace(prob, "cuda")
+    e = lambda *shape, dt=torch.bfloat16: torch.empty(*shape, device="cuda", dtype=dt)
+    W_s, W_t = torch.randn(V, d_s, device="cuda").bfloat16(), torch.randn(V, d_t, device="cuda").bfloat16()
+    f32 = lambda *shape: torch.empty(*shape, device="cuda")
+    dW = torch.full((V, d_s), float("nan"), device="cuda")
+    lib.opd_kl_fwd_bwd(prob, e(0, d_s), e(0, d_t), W_s, W_t, e(0, dt=torch.uint8), f32(0), f32(0), f32(0, 3),
+                       f32(0, d_s), dW, False, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    assert (dW == 0).all()
+    dW.fill_(2.0)
+    lib.opd_kl_fwd_bwd(prob, e(0, d_s), e(0, d_t), W_s, W_t, e(0, dt=torch.uint8), f32(0), f32(0), f32(0, 3),
+                       f32(0, d_s), dW, True, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    assert (dW == 2.0).all()
+    prob1 = lib.make_problem(0, d_s, d_s, V, lib.OPD_DTYPE_BF16, 1.0)
+    tok = torch.empty(0, device="cuda", dtype=torch.int32)
+    lib.opd_score_tokens(prob1, e(0, d_s), W_s, tok, e(0, dt=torch.uint8), f32(0), f32(0), ws)
+    dW.fill_(float("nan"))
+    lib.opd_surrogate_fwd_bwd(prob1, e(0, d_s), W_s, tok, f32(0), f32(0), e(0, dt=torch.uint8), f32(0), f32(0),
+                              f32(0), f32(0, d_s), dW, False, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    assert (dW == 0).all()
+
+
 def test_student_equals_teacher_gives_zero(lib):
     w = _small_bf16(T=256, d_t=256, seed=18)
     lay = synth.layout(w)
