@@ -330,6 +330,32 @@ def test_bounded_wait_timeout_reports_and_context_survives(lib):
 FULL = ["qwen3_0p6b", "qwen3_1p7b", "qwen3_4b", "ragged_multiturn"]
 
 
+def test_largest_batch_sampled_rows(lib, oracle_mod):
+    """T = 131,072 packed tokens (twice the ragged workload): dz alone is 40 GB, so byte offsets
+    pass 2^32; sampled rows against the oracle, which gets only those rows (rows are independent)."""
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="largest", T=131072, n_traj=256, seed=27)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    out = _run(lib, w, x, lay.mask, g)
+    sup = lay.mask != 0
+    assert (out["kl"][~sup] == 0).all() and (out["dH"][~sup] == 0).all() and np.isfinite(out["dW"]).all()
+    rows = np.flatnonzero(sup)
+    pick = np.unique(np.concatenate([rows[np.linspace(0, len(rows) - 1, 12).astype(int)], rows[-2:]]))
+    sel = torch.as_tensor(pick, device="cuda")
+    H_s, H_t = (synth.host_values(x[k].index_select(0, sel)) for k in ("H_s", "H_t"))
+    W_s, W_t = synth.host_values(x["W_s"]), synth.host_values(x["W_t"])
+    ones = np.ones(len(pick), np.uint8)
+    ref = oracle_mod.opd_kl(H_s, H_t, W_s, W_t, ones, _g64(g[pick], ones), w.tau)
+    _check_kl(out["kl"][pick], ref.kl)
+    assert _rel(out["dH"][pick], ref.dH_s) <= GRAD_REL
+    # dW_s at the same size with only the sampled rows supervised
+    mask2 = np.zeros_like(lay.mask)
+    mask2[pick] = 1
+    out2 = _run(lib, w, x, mask2, g)
+    assert _rel(out2["dW"], ref.dW_s) <= GRAD_REL, _rel(out2["dW"], ref.dW_s)
+
+
 @pytest.mark.parametrize("name", FULL)
 def test_full_size_sampled_rows(lib, oracle_mod, name):
     w = synth.WORKLOADS[name]
