@@ -345,10 +345,11 @@ opd_status forward_body(const Call& c, const Maps& m, float* kl_out, float* stat
   return OPD_OK;
 }
 
-opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s, int accumulate_dW);
+// dW_s is written through the tensor map m.dw (encoded over the caller's dW_s).
+opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumulate_dW);
 
 opd_status backward_body(const Call& c, const Maps& m, const float* stats, const float* grad_kl, float* dH_s,
-                         float* dW_s, int accumulate_dW) {
+                         int accumulate_dW) {
   FusedParams fp = fused_params(c);
   float4* rowc = reinterpret_cast<float4*>(c.ws + c.L.rowc);
   OPD_CUDA(timed("bwd_rowc", c.s, [&] {
@@ -357,12 +358,12 @@ opd_status backward_body(const Call& c, const Maps& m, const float* stats, const
   OPD_CUDA(timed("fused_logits_bwd", c.s, [&] {
     return launch_fused_backward(m.hs, m.ht, m.ws, m.wt, m.dz_store, fp, c.dev.sm_count, c.s);
   }));
-  return gradient_gemms(c, m, dH_s, dW_s, accumulate_dW);
+  return gradient_gemms(c, m, dH_s, accumulate_dW);
 }
 
 // dH_s = dZ W_s (split-K partial sums, then scattered back to the T rows) and
 // dW_s (+)= dZ^T H_s, from the bf16 dz the fused backward wrote.
-opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, float* dW_s, int accumulate_dW) {
+opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumulate_dW) {
   float* dhg = reinterpret_cast<float*>(c.ws + c.L.dh_g);
   OPD_CUDA(timed("zero_rows", c.s, [&] {
     return launch_zero_rows(dhg, (int32_t)c.p.d_s, c.ctrl(), (int32_t)c.L.T_pad, c.dev.sm_count, c.s);
@@ -444,7 +445,7 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
   Maps m;
   OPD_TRY(encode_maps(c, W_s, W_t, dW_s, m, do_bwd));
   if (do_fwd) OPD_TRY(forward_body(c, m, kl_out, stats_out));
-  if (do_bwd) OPD_TRY(backward_body(c, m, stats, grad_kl, dH_s, dW_s, accumulate_dW));
+  if (do_bwd) OPD_TRY(backward_body(c, m, stats, grad_kl, dH_s, accumulate_dW));
   return finish_call(c, outputs);
 }
 
@@ -501,7 +502,7 @@ opd_status head_call(const opd_problem* problem, const void* H, const void* W, c
   if (surrogate) {
     OPD_CUDA(timed("head_logits_bwd", c.s,
                    [&] { return launch_head_backward(m.hs, m.ws, m.dz_store, fp, c.dev.sm_count, c.s); }));
-    OPD_TRY(gradient_gemms(c, m, dH, dW, accumulate_dW));
+    OPD_TRY(gradient_gemms(c, m, dH, accumulate_dW));
   }
   Outputs outputs;
   const size_t Tn = (size_t)T;
