@@ -198,7 +198,7 @@ def test_out_of_range_token_is_reported_not_read(lib):
     assert lib.opd_kl_get_status(ws) == lib.OPD_OK
 
 
-@pytest.mark.parametrize("name", ["qwen3_1p7b"])
+@pytest.mark.parametrize("name", ["qwen3_0p6b", "qwen3_1p7b", "qwen3_4b", "ragged_multiturn"])
 def test_full_size_surrogate_and_scoring_sampled_rows(lib, oracle_mod, name):
     w = synth.WORKLOADS[name]
     lay = synth.layout(w)
