@@ -447,28 +447,45 @@ def run_gpu(args):
     ms_step = ms / args.steps
     value = whole_job_rate(R, args.steps, world, ms)
 
-    # end to end through the same C ABI: the step's inputs from pinned host memory, its
-    # per-token result back to the host every step
+    # end to end through the same C ABI: every step's inputs come from pinned host memory
+    # and its per-token result goes back to the host. Step i + 1's inputs are copied on a
+    # second stream, into the other of two device buffers, while step i computes.
     host_in = {k: v.cpu().pin_memory() for k, v in inputs.items()}
-    dev_in = {k: torch.empty_like(v) for k, v in inputs.items()}
+    dev_in = [{k: torch.empty_like(v) for k, v in inputs.items()} for _ in range(2)]
     res_h = torch.empty(result.shape, dtype=result.dtype).pin_memory()
     h2d = sum(t.numel() * t.element_size() for t in host_in.values())
     d2h = res_h.numel() * res_h.element_size()
+    compute, copier = torch.cuda.current_stream(), torch.cuda.Stream()
+    copied = [torch.cuda.Event(), torch.cuda.Event()]
+    consumed = [torch.cuda.Event(), torch.cuda.Event()]
 
-    def e2e_step():
-        for k, t in host_in.items():
-            dev_in[k].copy_(t, non_blocking=True)
-        step(dev_in)
-        res_h.copy_(result, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
-        return float(res_h.view(-1)[0])
+    def prefetch(b):
+        with torch.cuda.stream(copier):
+            copier.wait_event(consumed[b])  # the buffer's previous step has finished reading it
+            for k, t in host_in.items():
+                dev_in[b][k].copy_(t, non_blocking=True)
+            copied[b].record(copier)
 
-    e2e_step()
+    def e2e_steps(n):
+        for ev in consumed:  # copies of this run start after everything already on the compute stream
+            ev.record(compute)
+        prefetch(0)
+        for i in range(n):
+            b = i % 2
+            if i + 1 < n:
+                prefetch(1 - b)
+            compute.wait_event(copied[b])
+            step(dev_in[b])
+            consumed[b].record(compute)
+            res_h.copy_(result, non_blocking=True)
+            compute.synchronize()
+            float(res_h.view(-1)[0])
+
+    e2e_steps(1)
     barrier(world)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
-    for _ in range(args.steps):
-        e2e_step()
+    e2e_steps(args.steps)
     e1.record()
     torch.cuda.synchronize()
     barrier(world)
