@@ -132,6 +132,13 @@ def test_bf16_many_vocab_splits(lib, oracle_mod, tiling):
                                              seed=23))
 
 
+@pytest.mark.parametrize("tau", [0.1, 5.0])
+def test_bf16_extreme_temperatures(lib, oracle_mod, tau):
+    # tau = 0.1 spreads the scaled logits over hundreds of units (one token takes nearly all
+    # the mass); tau = 5 flattens both distributions
+    _full_check(lib, oracle_mod, _small_bf16(T=300, V=3000, tau=tau, n_traj=3, seed=28))
+
+
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
     w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
                     seed=13)
