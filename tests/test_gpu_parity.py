@@ -139,6 +139,31 @@ def test_bf16_extreme_temperatures(lib, oracle_mod, tau):
     _full_check(lib, oracle_mod, _small_bf16(T=300, V=3000, tau=tau, n_traj=3, seed=28))
 
 
+def _random_cases(n, seed=2026):
+    rng = np.random.default_rng(seed)
+    cases = []
+    for i in range(n):
+        cases.append(dict(T=int(rng.integers(1, 700)), d_s=8 * int(rng.integers(1, 41)), d_t=8 * int(rng.integers(1, 49)),
+                          V=int(rng.integers(2, 6000)), tau=float(rng.choice([0.3, 0.7, 1.0, 1.6])),
+                          density=float(rng.uniform(0.05, 1.0)), tiling=["bn256/cta1", "pair256/pair"][i % 2],
+                          seed=100 + i))
+    return cases
+
+
+@pytest.mark.parametrize("case", _random_cases(16), ids=lambda c: f"T{c['T']}-ds{c['d_s']}-dt{c['d_t']}-V{c['V']}")
+def test_random_shapes(lib, oracle_mod, case, monkeypatch):
+    """Seeded random problems: any T, hidden sizes in multiples of 8, any V, mixed temperatures and
+    mask densities, on both tilings."""
+    fused, gemm = case["tiling"].split("/")
+    monkeypatch.setenv("OPD_KL_FUSED", fused)
+    monkeypatch.setenv("OPD_KL_GEMM", gemm)
+    w = _small_bf16(T=case["T"], d_s=case["d_s"], d_t=case["d_t"], V=case["V"], tau=case["tau"], n_traj=1,
+                    traj_len=case["T"], seed=case["seed"])
+    mask = (np.random.default_rng(case["seed"]).random(w.T) < case["density"]).astype(np.uint8)
+    mask[np.random.default_rng(case["seed"] + 1).integers(0, w.T)] = 1
+    _full_check(lib, oracle_mod, w, mask=mask)
+
+
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
     w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
                     seed=13)
