@@ -227,6 +227,18 @@ def test_shapes_below_one_tile(lib, oracle_mod, shape, tiling):
     _full_check(lib, oracle_mod, w, mask=mask)
 
 
+@pytest.mark.parametrize("case", range(4))
+def test_fp32_random_shapes(lib, oracle_mod, case):
+    """The CUDA-core float32 path on seeded random small problems (any hidden size), tight bounds."""
+    rng = np.random.default_rng(300 + case)
+    w = synth.scaled(synth.WORKLOADS["tiny_fp32"], T=int(rng.integers(1, 120)), d_s=int(rng.integers(1, 96)),
+                     d_t=int(rng.integers(1, 160)), V=int(rng.integers(2, 1500)), tau=float(rng.uniform(0.5, 2.0)),
+                     seed=300 + case)
+    mask = (rng.random(w.T) < 0.7).astype(np.uint8)
+    mask[0] = 1
+    _full_check(lib, oracle_mod, w, mask=mask, tight=True)
+
+
 def test_fp32_two_token_vocabulary(lib, oracle_mod):
     w = synth.scaled(synth.WORKLOADS["tiny_fp32"], V=2, d_s=8, d_t=16, seed=22)
     _full_check(lib, oracle_mod, w, tight=True)

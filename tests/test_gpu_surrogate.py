@@ -161,6 +161,44 @@ def test_surrogate_and_scoring_below_one_tile(lib, oracle_mod, shape, tiling):
     assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
 
 
+def _random_cases(n, seed=4049):
+    rng = np.random.default_rng(seed)
+    return [dict(T=int(rng.integers(1, 600)), d_s=8 * int(rng.integers(1, 41)), V=int(rng.integers(2, 5000)),
+                 tau=float(rng.choice([0.4, 1.0, 1.7])), density=float(rng.uniform(0.1, 1.0)),
+                 tiling=["bn256/cta1", "pair256/pair"][i % 2], seed=200 + i) for i in range(n)]
+
+
+@pytest.mark.parametrize("case", _random_cases(8), ids=lambda c: f"T{c['T']}-d{c['d_s']}-V{c['V']}")
+def test_surrogate_and_scoring_random_shapes(lib, oracle_mod, case, monkeypatch):
+    fused, gemm = case["tiling"].split("/")
+    monkeypatch.setenv("OPD_KL_FUSED", fused)
+    monkeypatch.setenv("OPD_KL_GEMM", gemm)
+    w = _case(T=case["T"], d_s=case["d_s"], V=case["V"], tau=case["tau"], n_traj=1, traj_len=case["T"],
+              seed=case["seed"])
+    mask = (np.random.default_rng(case["seed"]).random(w.T) < case["density"]).astype(np.uint8)
+    mask[0] = 1
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    sup = mask != 0
+    lse, lp = _score(lib, w, x["H_s"], x["W_s"], tokens, mask)
+    ref_lse, ref_lp = oracle_mod.score(Hs, Ws, tokens, w.tau, rows=np.flatnonzero(sup))
+    _close(lse[sup], ref_lse, 1e-4, 1e-4, "lse")
+    _close(lp[sup], ref_lp, 1e-4, 1e-4, "logp")
+    _, lp_full = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = (lp_full - _clear_offsets(case["seed"], w.T)).astype(np.float32)
+    adv = np.random.default_rng(case["seed"] + 1).choice([-1.0, 1.0], w.T) * \
+        np.random.default_rng(case["seed"] + 2).uniform(0.2, 1.5, w.T)
+    logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
+    weights = np.where(sup, 1.0 / int(sup.sum()), 0.0).astype(np.float32)
+    loss, _, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, mask, weights)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               mask, weights.astype(np.float64), w.tau)
+    _close(loss, ref.loss, 1e-4, 2e-3, "loss")
+    assert _rel(dH, ref.dH_s) <= 1e-2, _rel(dH, ref.dH_s)
+    assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
+
+
 def test_surrogate_on_policy_and_accumulate(lib, oracle_mod):
     # rho = 1: the surrogate's gradient is the policy gradient -A (1[k = x] - p) / tau
     w = _case(T=300, d_s=128, V=2048, tau=1.0, n_traj=3, seed=33)
