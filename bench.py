@@ -611,7 +611,7 @@ def main():
                          "dual-clip surrogate; score: teacher token scoring")
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
     ap.add_argument("--cpu-rows-1t", type=int, default=4, help="rows of the one-core CPU-oracle sample")
-    ap.add_argument("--ref-rows", type=int, default=8, help="rows per step of --impl reference")
+    ap.add_argument("--ref-rows", type=int, default=16, help="rows per step of --impl reference (the oracle splits rows over the host cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--calibrate", type=float, default=0.0, metavar="SECONDS",
                     help="instead of the benchmark: sustained cuBLAS vs fused-step runs under the power cap")
