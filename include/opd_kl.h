@@ -114,6 +114,25 @@ opd_status opd_kl_fwd_bwd(const opd_problem* problem, const void* H_s, const voi
                           float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
                           void* stream);
 
+/* The paper's aggregation of the per-token KL into one batch loss (Appendix B.4: the
+ * seq-mean-token-mean of Eq. opd-surrogate, here applied to KL_i):
+ *   w_i = mask_i / (|B| (n_seg(i) + eps)),   L = sum_i w_i KL_i
+ * with n_b the supervised tokens of response b and |B| the distinct response ids. One call
+ * computes the weights on the device (as opd_seq_mean_token_mean_device), the forward
+ * with L summed inside its combine pass (in double, in no fixed order) and the backward
+ * with grad_kl = w. Writes loss_out[0] = L, kl_out [T], stats [T, 3], dH_s = dL/dH_s
+ * (zeros on masked rows) and dW_s = dL/dW_s (added to dW_s when accumulate_dW != 0).
+ * seg_id [T] int32: each row's response id, -1 outside responses; an id >= n_ids is
+ * skipped and reported by opd_kl_get_status as OPD_ERR_INVALID_ARG. The workspace holds
+ * opd_kl_seq_mean_workspace_size(problem, n_ids) bytes: the reverse-KL workspace, T
+ * weights and the response counters (0 for an invalid problem or n_ids < 1). */
+size_t opd_kl_seq_mean_workspace_size(const opd_problem* problem, int64_t n_ids);
+opd_status opd_kl_seq_mean_fwd_bwd(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                                   const void* W_t, const uint8_t* mask, const int32_t* seg_id, int64_t n_ids,
+                                   float eps, float* loss_out, float* kl_out, float* stats, float* dH_s,
+                                   float* dW_s, int accumulate_dW, void* workspace, size_t workspace_bytes,
+                                   void* stream);
+
 /* Token scoring under one head (the frozen teacher's scores, or the student's):
  * for every row with mask[i] = 1,
  *   lse_out[i]  = logsumexp_v (H[i,:] . W[v,:]) / temperature

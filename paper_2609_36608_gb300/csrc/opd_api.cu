@@ -333,13 +333,43 @@ FusedParams fused_params(const Call& c) {
   return fp;
 }
 
-opd_status forward_body(const Call& c, const Maps& m, float* kl_out, float* stats) {
+// The paper's batch loss over the per-token KL (Appendix B.4, seq-mean-token-mean):
+// per-token weights computed on the device, then L = sum_i w_i KL_i.
+struct SeqLoss {
+  const int32_t* seg_id;
+  int64_t n_ids;
+  float eps;
+  float* weights;  // [T] in the workspace; also the backward's upstream weights
+  void* scratch;   // seq-mean scratch (starts with the double accumulator of L)
+  float* loss_out; // [1]
+};
+
+// opd_kl_seq_mean_fwd_bwd's workspace: the reverse-KL workspace, then the per-token
+// weights, then the seq-mean scratch; 256-byte aligned sections.
+struct SeqLayout {
+  size_t weights = 0, scratch = 0, total = 0;
+};
+
+SeqLayout seq_layout(const WsLayout& L, int64_t n_ids) {
+  SeqLayout S;
+  size_t off = round_up(L.total, 256);
+  S.weights = off;
+  off = round_up(off + 4 * (size_t)L.T_pad, 256);
+  S.scratch = off;
+  off = round_up(off + seq_mean_token_mean_scratch_bytes(n_ids), 256);
+  S.total = off;
+  return S;
+}
+
+// Fused forward and combine; with loss weights, the combine also accumulates L.
+opd_status forward_body(const Call& c, const Maps& m, float* kl_out, float* stats, const SeqLoss* seq) {
   if (c.p.dtype == OPD_DTYPE_F32) return OPD_OK;  // handled by caller
   const FusedParams fp = fused_params(c);
   OPD_CUDA(timed("fused_logits_fwd", c.s,
                  [&] { return launch_fused_forward(m.hs, m.ht, m.ws, m.wt, fp, c.dev.sm_count, c.s); }));
   OPD_CUDA(timed("combine", c.s, [&] {
     return launch_combine(fp.partials, c.pos(), c.ctrl(), (int32_t)c.p.T, (int32_t)c.L.T_pad, kl_out, stats,
+                          seq ? seq->weights : nullptr, seq ? seq_mean_token_mean_acc(seq->scratch) : nullptr,
                           c.dev.sm_count, c.s);
   }));
   return OPD_OK;
@@ -404,7 +434,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumul
 opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s, const void* W_t,
                const uint8_t* mask, const float* grad_kl, float* kl_out, float* stats_out, const float* stats_in,
                float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t ws_bytes, void* stream,
-               bool do_fwd, bool do_bwd) {
+               bool do_fwd, bool do_bwd, const SeqLoss* seq = nullptr) {
   Call c;
   OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream));
   OPD_TRY(check_inputs(c, H_s, H_t, W_s, W_t, mask));
@@ -423,6 +453,13 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
   if (do_bwd) outputs.add(dH_s, Tn * (size_t)c.p.d_s).add(dW_s, (size_t)c.p.V * (size_t)c.p.d_s);
 
   OPD_TRY(prologue(c, H_s, H_t, mask));
+  if (seq) {  // the upstream weights of the batch loss, after compaction cleared the status word
+    OPD_CUDA(timed("seq_mean_token_mean", c.s, [&] {
+      return launch_seq_mean_token_mean(seq->seg_id, mask, (int32_t)T, (int32_t)seq->n_ids, seq->eps, nullptr,
+                                        seq->weights, nullptr, c.ctrl(), false, seq->scratch, c.dev.sm_count, c.s);
+    }));
+    outputs.add(seq->loss_out, 1);
+  }
   if (c.p.dtype == OPD_DTYPE_F32) {
     const float* hs = static_cast<const float*>(H_s);
     const float* ht = static_cast<const float*>(H_t);
@@ -432,6 +469,12 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
       OPD_CUDA(timed("simt_forward", c.s, [&] {
         return launch_simt_forward(hs, ht, ws, wt, (int32_t)T, (int32_t)c.p.d_s, (int32_t)c.p.d_t, (int32_t)c.p.V,
                                    c.p.temperature, c.idx(), c.pos(), c.ctrl(), kl_out, stats_out, c.s);
+      }));
+    if (seq)  // L from the forward's per-token KL (the CUDA-core path has no combine pass)
+      OPD_CUDA(timed("seq_mean_token_mean", c.s, [&] {
+        return launch_seq_mean_token_mean(seq->seg_id, mask, (int32_t)T, (int32_t)seq->n_ids, seq->eps, kl_out,
+                                          nullptr, seq->loss_out, c.ctrl(), false, seq->scratch, c.dev.sm_count,
+                                          c.s);
       }));
     if (do_bwd)
       OPD_CUDA(timed("simt_backward", c.s, [&] {
@@ -444,7 +487,10 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
 
   Maps m;
   OPD_TRY(encode_maps(c, W_s, W_t, dW_s, m, do_bwd));
-  if (do_fwd) OPD_TRY(forward_body(c, m, kl_out, stats_out));
+  if (do_fwd) OPD_TRY(forward_body(c, m, kl_out, stats_out, seq));
+  if (seq)
+    OPD_CUDA(timed("store_loss", c.s,
+                   [&] { return launch_store_loss(seq_mean_token_mean_acc(seq->scratch), seq->loss_out, c.s); }));
   if (do_bwd) OPD_TRY(backward_body(c, m, stats, grad_kl, dH_s, accumulate_dW));
   return finish_call(c, outputs);
 }
@@ -587,9 +633,29 @@ opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t*
   return OPD_OK;
 }
 
+size_t opd_kl_seq_mean_workspace_size(const opd_problem* problem, int64_t n_ids) {
+  if (check_problem(problem) != OPD_OK || n_ids < 1 || n_ids > (int64_t)0x7FFF0000) return 0;
+  return seq_layout(ws_layout(*problem), n_ids).total;
+}
+
+opd_status opd_kl_seq_mean_fwd_bwd(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
+                                   const void* W_t, const uint8_t* mask, const int32_t* seg_id, int64_t n_ids,
+                                   float eps, float* loss_out, float* kl_out, float* stats, float* dH_s, float* dW_s,
+                                   int accumulate_dW, void* workspace, size_t workspace_bytes, void* stream) {
+  OPD_TRY(check_problem(problem));
+  if (n_ids < 1 || n_ids > (int64_t)0x7FFF0000 || !(eps >= 0.0f) || !loss_out) return OPD_ERR_INVALID_ARG;
+  if (problem->T > 0 && !seg_id) return OPD_ERR_INVALID_ARG;
+  const SeqLayout S = seq_layout(ws_layout(*problem), n_ids);
+  if (!workspace || !aligned(workspace, 256) || workspace_bytes < S.total) return OPD_ERR_INVALID_ARG;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  SeqLoss seq{seg_id, n_ids, eps, reinterpret_cast<float*>(ws + S.weights), ws + S.scratch, loss_out};
+  return run(problem, H_s, H_t, W_s, W_t, mask, seq.weights, kl_out, stats, nullptr, dH_s, dW_s, accumulate_dW,
+             workspace, workspace_bytes, stream, true, true, &seq);
+}
+
 size_t opd_seq_mean_token_mean_workspace_size(int64_t n_ids) {
   if (n_ids < 1 || n_ids > (int64_t)0x7FFF0000) return 0;
-  return round_up(seq_mean_token_mean_scratch_bytes(n_ids), 256);
+  return round_up(sizeof(Ctrl) + seq_mean_token_mean_scratch_bytes(n_ids), 256);
 }
 
 opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* mask, int64_t T, int64_t n_ids,
@@ -606,7 +672,8 @@ opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   OPD_CUDA(timed("seq_mean_token_mean", s, [&] {
     return launch_seq_mean_token_mean(seg_id, mask, (int32_t)T, (int32_t)n_ids, eps, loss_in, w_out,
-                                      loss_in ? loss_out : nullptr, workspace, dev.sm_count, s);
+                                      loss_in ? loss_out : nullptr, static_cast<Ctrl*>(workspace), true,
+                                      static_cast<uint8_t*>(workspace) + sizeof(Ctrl), dev.sm_count, s);
   }));
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
   if (env_flag("OPD_KL_SYNC_CHECK")) {

@@ -94,9 +94,10 @@ __global__ void k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict_
 // then  lse = (M + log2 S) ln 2,  KL = (A_s / S_s) ln 2 - lse_s + lse_t.
 __global__ void k_combine(const float* __restrict__ part, const int32_t* __restrict__ pos,
                           const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
-                          float* __restrict__ stats) {
+                          float* __restrict__ stats, const float* __restrict__ weights, double* loss_acc) {
   const int n_vs = ctrl->n_vsplit;
   const size_t plane = (size_t)T_pad;
+  double wkl = 0.0;  // this thread's share of sum_i w_i KL_i (weights given)
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
     const int r = pos[i];
     float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
@@ -124,6 +125,12 @@ __global__ void k_combine(const float* __restrict__ part, const int32_t* __restr
     stats[3 * (size_t)i + 0] = lse_s;
     stats[3 * (size_t)i + 1] = lse_t;
     stats[3 * (size_t)i + 2] = kl;
+    if (weights && r >= 0) wkl += (double)weights[i] * (double)kl;
+  }
+  if (weights) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) wkl += __shfl_xor_sync(0xffffffffu, wkl, o);
+    if ((threadIdx.x & 31) == 0 && wkl != 0.0) atomicAdd(loss_acc, wkl);
   }
 }
 
@@ -206,8 +213,10 @@ cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, in
 }
 
 cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
-                           float* kl_out, float* stats, int n_sm, cudaStream_t s) {
-  k_combine<<<grid_for(T, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats);
+                           float* kl_out, float* stats, const float* weights, double* loss_acc, int n_sm,
+                           cudaStream_t s) {
+  k_combine<<<grid_for(T, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats, weights,
+                                                   loss_acc);
   return cudaGetLastError();
 }
 

@@ -81,8 +81,10 @@ cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t
                            cudaStream_t s);
 cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, int32_t d_t, const int32_t* idx,
                                const Ctrl* ctrl, void* Hs_g, void* Ht_g, int32_t T_pad, int n_sm, cudaStream_t s);
+// weights != nullptr: also adds sum_i weights[i] KL_i to *loss_acc (the batch loss, fused here).
 cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
-                           float* kl_out, float* stats, int n_sm, cudaStream_t s);
+                           float* kl_out, float* stats, const float* weights, double* loss_acc, int n_sm,
+                           cudaStream_t s);
 cudaError_t launch_bwd_rowc(const float* stats, const float* grad_kl, const int32_t* idx, const Ctrl* ctrl,
                             int32_t T_pad, float tau, float4* rowc, cudaStream_t s);
 cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t T_pad, int n_sm, cudaStream_t s);
@@ -116,11 +118,15 @@ cudaError_t launch_head_forward(const CUtensorMap& h, const CUtensorMap& w, cons
 cudaError_t launch_head_backward(const CUtensorMap& h, const CUtensorMap& w, const CUtensorMap& dz_store,
                                  const FusedParams& p, int grid, cudaStream_t s);
 cudaError_t launch_head_rows(const HeadRowsParams& p, int n_sm, cudaStream_t s);
-// seq-mean-token-mean on the device (opd_seqmean.cu); workspace starts with a Ctrl.
+// seq-mean-token-mean on the device (opd_seqmean.cu). Scratch of seq_mean_token_mean_scratch_bytes
+// (starts with the double loss accumulator); bad response ids set ctrl->status, which the first
+// kernel clears when clear_status is set.
 size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids);
+double* seq_mean_token_mean_acc(void* scratch);
 cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, float eps,
-                                       const float* loss_in, float* w_out, float* loss_out, void* workspace,
-                                       int n_sm, cudaStream_t s);
+                                       const float* loss_in, float* w_out, float* loss_out, Ctrl* ctrl,
+                                       bool clear_status, void* scratch, int n_sm, cudaStream_t s);
+cudaError_t launch_store_loss(const double* acc, float* loss_out, cudaStream_t s);
 // C = A * B^T with A [M, K] and B [N, K] given through tensor maps; a_mn / b_mn select
 // MN-major operand tiles (the operand's contiguous dimension is M or N, not K).
 cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,

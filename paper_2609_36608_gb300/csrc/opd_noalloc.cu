@@ -152,7 +152,8 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.max_vsplit = kSplits;
   fp.rowc = nullptr;
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
-  if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
+  if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
+    return OPD_ERR_CUDA;
 
   const char* sync = std::getenv("OPD_KL_SYNC_CHECK");
   if (sync && sync[0] && sync[0] != '0') {

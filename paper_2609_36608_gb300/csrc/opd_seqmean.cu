@@ -12,15 +12,16 @@ namespace opd {
 
 namespace {
 
-// Workspace: Ctrl (status), then [double acc][int32 n_resp, pad][counts n_ids][present n_ids].
-__global__ void k_seq_zero(Ctrl* ctrl, int32_t* counts, int32_t* present, int32_t n_ids, int32_t* n_resp,
-                           double* acc) {
+// Scratch: [double acc][int32 n_resp, pad][counts n_ids][present n_ids]; the status word
+// lives in a Ctrl of the caller's workspace.
+__global__ void k_seq_zero(uint32_t* status, bool clear_status, int32_t* counts, int32_t* present, int32_t n_ids,
+                           int32_t* n_resp, double* acc) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_ids; i += gridDim.x * blockDim.x) {
     counts[i] = 0;
     present[i] = 0;
   }
   if (blockIdx.x == 0 && threadIdx.x == 0) {
-    ctrl->status = 0u;
+    if (clear_status) *status = 0u;
     *n_resp = 0;
     *acc = 0.0;
   }
@@ -71,13 +72,23 @@ __global__ void k_seq_store(const double* acc, float* loss_out) { *loss_out = (f
 
 }  // namespace
 
-size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids) { return sizeof(Ctrl) + 16 + 8 * (size_t)n_ids; }
+cudaError_t launch_store_loss(const double* acc, float* loss_out, cudaStream_t s) {
+  k_seq_store<<<1, 1, 0, s>>>(acc, loss_out);
+  return cudaGetLastError();
+}
+
+namespace {
+
+}  // namespace
+
+size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids) { return 16 + 8 * (size_t)n_ids; }
+
+double* seq_mean_token_mean_acc(void* scratch) { return static_cast<double*>(scratch); }
 
 cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, float eps,
-                                       const float* loss_in, float* w_out, float* loss_out, void* workspace,
-                                       int n_sm, cudaStream_t s) {
-  Ctrl* ctrl = static_cast<Ctrl*>(workspace);
-  double* acc = reinterpret_cast<double*>(static_cast<uint8_t*>(workspace) + sizeof(Ctrl));
+                                       const float* loss_in, float* w_out, float* loss_out, Ctrl* ctrl,
+                                       bool clear_status, void* scratch, int n_sm, cudaStream_t s) {
+  double* acc = static_cast<double*>(scratch);
   int32_t* n_resp = reinterpret_cast<int32_t*>(acc + 1);
   int32_t* counts = n_resp + 2;
   int32_t* present = counts + n_ids;
@@ -88,7 +99,7 @@ cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, 
     if (b > (long)n_sm * 4) b = (long)n_sm * 4;
     return (int)(b < 1 ? 1 : b);
   };
-  k_seq_zero<<<blocks(n_ids), threads, 0, s>>>(ctrl, counts, present, n_ids, n_resp, acc);
+  k_seq_zero<<<blocks(n_ids), threads, 0, s>>>(status, clear_status, counts, present, n_ids, n_resp, acc);
   k_seq_hist<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, present, status);
   k_seq_count<<<blocks(n_ids), threads, 0, s>>>(present, n_ids, n_resp);
   k_seq_weights<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, n_resp, eps, loss_in, w_out, acc);

@@ -70,6 +70,9 @@ def _load() -> ctypes.CDLL:
         "opd_surrogate_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, vp, ctypes.POINTER(opd_surrogate_params),
                                         vp, vp, vp, vp, i32, vp, sz, vp]),
         "opd_seq_mean_token_mean_workspace_size": (sz, [i64]),
+        "opd_kl_seq_mean_workspace_size": (sz, [P, i64]),
+        "opd_kl_seq_mean_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, i64, ctypes.c_float, vp, vp, vp, vp, vp, i32,
+                                          vp, sz, vp]),
         "opd_seq_mean_token_mean_device": (i32, [vp, vp, i64, i64, ctypes.c_float, vp, vp, vp, vp, sz, vp]),
         "opd_kl_profile_start": (i32, []),
         "opd_kl_profile_stop": (i32, [ctypes.POINTER(opd_kernel_time), i32, ctypes.POINTER(i32)]),
@@ -158,6 +161,28 @@ def opd_kl_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, grad_kl, kl_out, stats, dH
                                _ptr(grad_kl), _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s),
                                int(bool(accumulate_dW)), _ptr(workspace), workspace.numel(), _stream(stream)),
            "opd_kl_fwd_bwd")
+
+
+def opd_kl_seq_mean_workspace_size(problem, n_ids: int) -> int:
+    return int(_lib.opd_kl_seq_mean_workspace_size(ctypes.byref(problem), int(n_ids)))
+
+
+def allocate_seq_mean_workspace(problem, n_ids: int, device="cuda") -> torch.Tensor:
+    n = opd_kl_seq_mean_workspace_size(problem, n_ids)
+    if n == 0:
+        raise ValueError("invalid problem or n_ids")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def opd_kl_seq_mean_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, seg_id, n_ids: int, eps: float, loss_out, kl_out,
+                            stats, dH_s, dW_s, accumulate_dW: bool, workspace, stream=None) -> None:
+    """The paper's batch loss over the per-token KL (seq-mean-token-mean weights on the device, L summed
+    in the combine pass) and its gradients, in one call."""
+    _check(_lib.opd_kl_seq_mean_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t),
+                                        _ptr(mask), _ptr(seg_id), int(n_ids), float(eps), _ptr(loss_out),
+                                        _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
+                                        _ptr(workspace), workspace.numel(), _stream(stream)),
+           "opd_kl_seq_mean_fwd_bwd")
 
 
 def opd_score_tokens(problem, H, W, tokens, mask, lse_out, logp_out, workspace, stream=None) -> None:

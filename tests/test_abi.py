@@ -106,3 +106,22 @@ def test_seq_mean_token_mean_device_arguments(lib):
     rc = lib.call_raw("opd_seq_mean_token_mean_device", fake, fake, ctypes.c_int64(4), ctypes.c_int64(2),
                       ctypes.c_float(-1.0), None, fake, None, fake, ctypes.c_size_t(4096), None)
     assert rc == lib.OPD_ERR_INVALID_ARG
+
+
+def test_kl_seq_mean_arguments(lib):
+    p = lib.make_problem(1000, 64, 64, 500, lib.OPD_DTYPE_BF16, 1.0)
+    base = lib.opd_kl_workspace_size(p)
+    assert lib.opd_kl_seq_mean_workspace_size(p, 10) >= base + 4 * 1000 + 16 + 80
+    assert lib.opd_kl_seq_mean_workspace_size(p, 0) == 0
+    assert lib.opd_kl_seq_mean_workspace_size(lib.make_problem(8, 12, 8, 8), 4) == 0
+    vp = ctypes.c_void_p
+    fake = vp(1 << 20)
+    n = ctypes.c_size_t(lib.opd_kl_seq_mean_workspace_size(p, 10))
+    args = lambda n_ids, eps, loss: [ctypes.byref(p), fake, fake, fake, fake, fake, fake, ctypes.c_int64(n_ids),
+                                     ctypes.c_float(eps), loss, fake, fake, fake, fake, 0, fake, n, None]
+    assert lib.call_raw("opd_kl_seq_mean_fwd_bwd", *args(0, 1e-8, fake)) == lib.OPD_ERR_INVALID_ARG
+    assert lib.call_raw("opd_kl_seq_mean_fwd_bwd", *args(10, -1.0, fake)) == lib.OPD_ERR_INVALID_ARG
+    assert lib.call_raw("opd_kl_seq_mean_fwd_bwd", *args(10, 1e-8, None)) == lib.OPD_ERR_INVALID_ARG
+    small = [ctypes.byref(p), fake, fake, fake, fake, fake, fake, ctypes.c_int64(10), ctypes.c_float(1e-8), fake,
+             fake, fake, fake, fake, 0, fake, ctypes.c_size_t(base), None]
+    assert lib.call_raw("opd_kl_seq_mean_fwd_bwd", *small) == lib.OPD_ERR_INVALID_ARG  # KL workspace only
