@@ -189,7 +189,8 @@ def source_hash(name):
 def recorded_traffic(name, workload, step_path="kl"):
     """DRAM bytes per launch from the committed ncu summary, if the kernel source still matches
     (profiles/<kernel>_<workload>.txt for the KL step, <kernel>_<path>_<workload>.txt otherwise)."""
-    tag = workload if step_path == "kl" else f"{step_path}_{workload}"
+    # the loss step runs the reverse-KL step's kernels on the same shapes
+    tag = workload if step_path in ("kl", "kl_seqmean") else f"{step_path}_{workload}"
     path = os.path.join(ROOT, "profiles", f"{name}_{tag}.txt")
     if not os.path.exists(path):
         return None
@@ -243,7 +244,7 @@ def run_reference(args):
     tokens = synth.token_ids(w.seed, w.T, w.V)
 
     def one(rows):
-        if args.path == "kl":
+        if args.path in ("kl", "kl_seqmean"):
             oracle_rate(w, host, lay, g, rows, threads)
         elif args.path == "score":
             oracle.score(host["H_t"], host["W_t"], tokens, w.tau, rows=rows, n_threads=threads)
@@ -262,6 +263,7 @@ def run_reference(args):
     dt = time.perf_counter() - t0
     value = n / dt
     what = {"kl": "logits, KL, dH_s rows and their dW_s contribution",
+            "kl_seqmean": "logits, KL, dH_s rows and their dW_s contribution (seq-mean-token-mean weights)",
             "score": "teacher log-partition and token log-probabilities",
             "surrogate": "student logits, dual-clip loss, dH_s rows and their dW_s contribution"}[args.path]
     sample = (f"{rows_per_step} supervised rows of {w.name} per step (full V={w.V}, d_s={w.d_s}, d_t={w.d_t}): "
@@ -283,6 +285,7 @@ PATH_METRICS = {
     "kl": METRIC,
     "surrogate": "response tokens/s, sampled-token dual-clip surrogate loss step fwd+bwd (1 GB300)",
     "score": "response tokens/s, teacher token scoring fwd (1 GB300)",
+    "kl_seqmean": "response tokens/s, fused OPD KL loss step (seq-mean-token-mean on the device) fwd+bwd (1 GB300)",
 }
 
 
@@ -305,6 +308,20 @@ def path_setup(path, w, lay, x, dev, opd_kl):
                                   dW, False, ws)
         executed, algorithmic = step_flops(w, R)
         return inputs, step, kl, ws, executed, algorithmic
+    if path == "kl_seqmean":
+        # the whole loss step: weights from response ids on the device, L = sum_i w_i KL_i, gradients of L
+        prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
+        n_ids = int(lay.seg_id.max()) + 1
+        ws = opd_kl.allocate_seq_mean_workspace(prob, n_ids, dev)
+        loss, kl, stats = torch.empty(1, device=dev), torch.empty(w.T, device=dev), torch.empty(w.T, 3, device=dev)
+        dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+        inputs = {"H_s": x["H_s"], "H_t": x["H_t"], "mask": mask, "seg_id": torch.from_numpy(lay.seg_id).to(dev)}
+
+        def step(i):
+            opd_kl.opd_kl_seq_mean_fwd_bwd(prob, i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["seg_id"],
+                                           n_ids, 1e-8, loss, kl, stats, dH, dW, False, ws)
+        executed, algorithmic = step_flops(w, R)
+        return inputs, step, loss, ws, executed, algorithmic
     tokens = torch.from_numpy(synth.token_ids(w.seed, w.T, w.V)).to(dev)
     if path == "score":
         prob = opd_kl.make_problem(w.T, w.d_t, w.d_t, w.V, dtype, w.tau)
@@ -341,7 +358,7 @@ def path_setup(path, w, lay, x, dev, opd_kl):
 
 
 def path_kernel_flops(path, name, w, R):
-    if path == "kl":
+    if path in ("kl", "kl_seqmean"):
         return kernel_flops(name, w, R)
     d = w.d_t if path == "score" else w.d_s
     if name in ("head_logits_fwd", "head_logits_bwd"):
@@ -358,7 +375,7 @@ def path_cpu_baseline(path, w, lay, x, args):
     oracle.build()
     threads = os.cpu_count() or 1
     rows = sample_rows(lay.mask, args.cpu_rows, 3)
-    if path == "kl":
+    if path in ("kl", "kl_seqmean"):
         host = host_inputs(x)
         g = np.where(lay.mask != 0, opd_seq_weights(lay), 0.0)
 
