@@ -92,46 +92,60 @@ __global__ void k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict_
 // Merge the base-2 statistics of every vocabulary split of one row:
 //   M = max_j m_j,  S = sum_j S_j 2^(m_j - M),  A likewise
 // then  lse = (M + log2 S) ln 2,  KL = (A_s / S_s) ln 2 - lse_s + lse_t.
+// Merge of two base-2 partial statistics (max M, sum S at M, A at M for the student;
+// the teacher's max and sum) into the first.
+__device__ __forceinline__ void merge_partial(float& ms, float& ss, float& as, float& mt, float& st, float ms2,
+                                              float ss2, float as2, float mt2, float st2) {
+  const float Ms = fmaxf(ms, ms2), Mt = fmaxf(mt, mt2);
+  const float f1 = ms == -CUDART_INF_F ? 0.f : exp2f(ms - Ms), f2 = ms2 == -CUDART_INF_F ? 0.f : exp2f(ms2 - Ms);
+  const float g1 = mt == -CUDART_INF_F ? 0.f : exp2f(mt - Mt), g2 = mt2 == -CUDART_INF_F ? 0.f : exp2f(mt2 - Mt);
+  ss = ss * f1 + ss2 * f2;
+  as = as * f1 + as2 * f2;
+  st = st * g1 + st2 * g2;
+  ms = Ms;
+  mt = Mt;
+}
+
+// One warp per token row: the lanes take the vocabulary splits' partials, then merge
+// them by shuffles. With weights, sum_i weights[i] KL_i is also added to *loss_acc.
 __global__ void k_combine(const float* __restrict__ part, const int32_t* __restrict__ pos,
                           const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
                           float* __restrict__ stats, const float* __restrict__ weights, double* loss_acc) {
   const int n_vs = ctrl->n_vsplit;
   const size_t plane = (size_t)T_pad;
-  double wkl = 0.0;  // this thread's share of sum_i w_i KL_i (weights given)
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+  const int lane = threadIdx.x & 31;
+  const int warps = (gridDim.x * blockDim.x) >> 5;
+  double wkl = 0.0;  // lane 0's share of sum_i w_i KL_i
+  for (int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < T; i += warps) {
     const int r = pos[i];
     float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
     if (r >= 0 && n_vs > 0) {
-      float Ms = -CUDART_INF_F, Mt = -CUDART_INF_F;
-      for (int j = 0; j < n_vs; ++j) {
+      float ms = -CUDART_INF_F, ss = 0.f, as = 0.f, mt = -CUDART_INF_F, st = 0.f;
+      for (int j = lane; j < n_vs; j += 32) {
         const float* b = part + (size_t)j * 5 * plane + r;
-        Ms = fmaxf(Ms, b[0]);
-        Mt = fmaxf(Mt, b[3 * plane]);
+        merge_partial(ms, ss, as, mt, st, b[0], b[plane], b[2 * plane], b[3 * plane], b[4 * plane]);
       }
-      float Ss = 0.f, As = 0.f, St = 0.f;
-      for (int j = 0; j < n_vs; ++j) {
-        const float* b = part + (size_t)j * 5 * plane + r;
-        const float fs = exp2f(b[0] - Ms);
-        Ss = fmaf(b[plane], fs, Ss);
-        As = fmaf(b[2 * plane], fs, As);
-        St = fmaf(b[4 * plane], exp2f(b[3 * plane] - Mt), St);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ms2 = __shfl_xor_sync(0xffffffffu, ms, o), ss2 = __shfl_xor_sync(0xffffffffu, ss, o);
+        const float as2 = __shfl_xor_sync(0xffffffffu, as, o), mt2 = __shfl_xor_sync(0xffffffffu, mt, o);
+        const float st2 = __shfl_xor_sync(0xffffffffu, st, o);
+        merge_partial(ms, ss, as, mt, st, ms2, ss2, as2, mt2, st2);
       }
       const float ln2 = 0.69314718055994531f;
-      lse_s = (Ms + log2f(Ss)) * ln2;
-      lse_t = (Mt + log2f(St)) * ln2;
-      kl = (As / Ss) * ln2 - lse_s + lse_t;
+      lse_s = (ms + log2f(ss)) * ln2;
+      lse_t = (mt + log2f(st)) * ln2;
+      kl = (as / ss) * ln2 - lse_s + lse_t;
     }
-    kl_out[i] = kl;
-    stats[3 * (size_t)i + 0] = lse_s;
-    stats[3 * (size_t)i + 1] = lse_t;
-    stats[3 * (size_t)i + 2] = kl;
-    if (weights && r >= 0) wkl += (double)weights[i] * (double)kl;
+    if (lane == 0) {
+      kl_out[i] = kl;
+      stats[3 * (size_t)i + 0] = lse_s;
+      stats[3 * (size_t)i + 1] = lse_t;
+      stats[3 * (size_t)i + 2] = kl;
+      if (weights && r >= 0) wkl += (double)weights[i] * (double)kl;
+    }
   }
-  if (weights) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) wkl += __shfl_xor_sync(0xffffffffu, wkl, o);
-    if ((threadIdx.x & 31) == 0 && wkl != 0.0) atomicAdd(loss_acc, wkl);
-  }
+  if (weights && lane == 0 && wkl != 0.0) atomicAdd(loss_acc, wkl);
 }
 
 __global__ void k_bwd_rowc(const float* __restrict__ stats, const float* __restrict__ grad_kl,
@@ -215,8 +229,8 @@ cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, in
 cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
                            float* kl_out, float* stats, const float* weights, double* loss_acc, int n_sm,
                            cudaStream_t s) {
-  k_combine<<<grid_for(T, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats, weights,
-                                                   loss_acc);
+  k_combine<<<grid_for((long)T * 32, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats,
+                                                               weights, loss_acc);
   return cudaGetLastError();
 }
 
