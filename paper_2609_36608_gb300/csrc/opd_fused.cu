@@ -296,23 +296,20 @@ __device__ __forceinline__ void fwd_chunk1(uint32_t ts, int nvalid_base, float k
 }
 
 // One head, backward of a loss on the sampled token's log-probability:
-// dz = coef (1[col = x] - p), p = 2^(z k2 - b1); bf16 into the warp's staging box.
+// dz = coef (1[col = x] - p), p = 2^(z k2 - b1), into the warp's staging box. This writes
+// -coef p in every column; token_fixup() then puts coef (1 - p_x) in the token's column.
 template <int C>
-__device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, float coef, int x_rel, uint32_t stg,
-                                           int lane) {
+__device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, float coef, uint32_t stg, int lane) {
   uint32_t rs[32];
   tmem_ld32(ts + C * 32, rs);
   uint32_t w[16];
-  const uint64_t k22 = f2_pack(k2, k2), nb2 = f2_pack(-b1, -b1), coef2 = f2_pack(coef, coef);
+  const uint64_t k22 = f2_pack(k2, k2), nb2 = f2_pack(-b1, -b1), ncoef2 = f2_pack(-coef, -coef);
 #pragma unroll
   for (int j = 0; j < 16; ++j) {
-    // two columns per instruction: dz = coef (1[col = x] - p), p = 2^(z k2 - b1)
-    const int col = C * 32 + 2 * j;
+    // two columns per instruction: -coef 2^(z k2 - b1)
     float a, b;
     f2_unpack(f2_fma(f2_pack(__uint_as_float(rs[2 * j]), __uint_as_float(rs[2 * j + 1])), k22, nb2), a, b);
-    const uint64_t p = f2_pack(ex2_ftz(a), ex2_ftz(b));
-    const uint64_t hot = f2_pack(col == x_rel ? 1.0f : 0.0f, col + 1 == x_rel ? 1.0f : 0.0f);
-    f2_unpack(f2_mul(coef2, f2_sub(hot, p)), a, b);
+    f2_unpack(f2_mul(ncoef2, f2_pack(ex2_ftz(a), ex2_ftz(b))), a, b);
     w[j] = pack_bf16x2(a, b);
   }
   const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
@@ -321,6 +318,15 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
   for (int jj = 0; jj < 4; ++jj)
     st_shared_v4(box + sw128_offset((uint32_t)lane, jb + jj), w[4 * jj], w[4 * jj + 1], w[4 * jj + 2],
                  w[4 * jj + 3]);
+}
+
+// The token's column of one row in a 64-column staging box (128-byte swizzled rows,
+// one row per lane): overwritten with the bf16 of `value` when the token lies in it.
+__device__ __forceinline__ void token_fixup(uint32_t box, int lane, int col_in_box, float value) {
+  if (col_in_box < 0 || col_in_box >= 64) return;
+  const uint32_t addr = box + sw128_offset((uint32_t)lane, (uint32_t)(col_in_box >> 3)) + (uint32_t)(col_in_box & 7) * 2u;
+  const __nv_bfloat16 h = __float2bfloat16_rn(value);
+  asm volatile("st.shared.b16 [%0], %1;" ::"r"(addr), "h"(*reinterpret_cast<const unsigned short*>(&h)) : "memory");
 }
 
 template <bool BWD, bool PAIR, int HEADS>
@@ -588,8 +594,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int row = row_base + row_in_tile;
       float ms = -INFINITY, Ss = 0.f, A = 0.f, mt = -INFINITY, St = 0.f;
       // backward row constants. Two heads: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc).
-      // One head: dz = coef (1[col = x] - p_s) with coef = rowc.y and token x = rowc.z (bits).
-      float b1 = 0.f, kc = 0.f, cc = 0.f;
+      // One head: dz = coef (1[col = x] - p_s) with coef = rowc.y, token x = rowc.z (bits) and
+      // the token column's value coef (1 - p_x) = rowc.w.
+      float b1 = 0.f, kc = 0.f, cc = 0.f, at_token = 0.f;
       int x_tok = -1;
       if (BWD) {
         const float4 rc = p.rowc[row];
@@ -600,6 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           kc = rc.y;
           x_tok = __float_as_int(rc.z);
+          at_token = rc.w;
         }
       }
       for (int vt = vb; vt < ve; ++vt, ++lt) {
@@ -626,8 +634,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int x_rel = x_tok - col0;  // the token's column within this warp's 128
             if (lane == 0) bulk_wait_read<1>();
             __syncwarp();
-            bwd_chunk1<0>(ts, p.k2, b1, kc, x_rel, stg, lane);
-            bwd_chunk1<1>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            bwd_chunk1<0>(ts, p.k2, b1, kc, stg, lane);
+            bwd_chunk1<1>(ts, p.k2, b1, kc, stg, lane);
+            token_fixup(stg, lane, x_rel, at_token);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
@@ -636,8 +645,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               bulk_wait_read<1>();
             }
             __syncwarp();
-            bwd_chunk1<2>(ts, p.k2, b1, kc, x_rel, stg, lane);
-            bwd_chunk1<3>(ts, p.k2, b1, kc, x_rel, stg, lane);
+            bwd_chunk1<2>(ts, p.k2, b1, kc, stg, lane);
+            bwd_chunk1<3>(ts, p.k2, b1, kc, stg, lane);
+            token_fixup(stg + 4096u, lane, x_rel - 64, at_token);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {

@@ -12,7 +12,8 @@
 //   l_clip = -min(rho A, clip(rho, 1 - delta, 1 + delta) A)
 //   l_DC  = min(l_clip, -kappa A) if A < 0 else l_clip
 //   coef_i = w_i (d l_DC / d logp_i) / tau,  so that the backward emits
-//   dz_i[k] = coef_i (1[k = x_i] - p_i[k]).
+//   dz_i[k] = coef_i (1[k = x_i] - p_i[k]); rowc carries coef_i (1 - p_i[x_i]) for the
+//   token's column, with p_i[x_i] = exp(logp_i).
 #include <math_constants.h>
 
 #include "opd_device.cuh"
@@ -122,7 +123,9 @@ __global__ void k_head_rows(const HeadRowsParams p) {
         if (x_ok) dual_clip(logp, p.logp_old[i], A, p.delta, p.kappa, p.clip, loss, slope);
         p.loss_out[i] = loss;
         const float coef = p.weights[i] * slope * p.inv_tau;
-        p.rowc[r] = make_float4(lse * 1.4426950408889634f, coef, __int_as_float(x), 0.f);
+        // the backward writes -coef p everywhere and this value, coef (1 - p_x), at the token
+        const float at_token = x_ok ? coef * (1.0f - expf(logp)) : 0.f;
+        p.rowc[r] = make_float4(lse * 1.4426950408889634f, coef, __int_as_float(x), at_token);
       }
     }
   }
