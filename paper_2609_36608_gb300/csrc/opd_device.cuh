@@ -161,6 +161,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32
   }
 }
 
+// Bounded wait without the early exit on a raised status: used only while draining
+// copies or MMAs already in flight before a CTA exits.
+__device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  const uint32_t addr = smem_u32(bar);
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 0; !mbar_try_wait(addr, parity); ++it) {
+    if ((it & 63u) == 63u && (globaltimer_ns() - t0 > limit_ns || it >= (1u << 28))) return;
+  }
+}
+
 // --------------------------------------------------------------------- TMA --
 
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, uint64_t* bar, int32_t c0,

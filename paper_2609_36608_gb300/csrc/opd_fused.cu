@@ -122,15 +122,6 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-// Wait without the early exit on a raised status: used only while draining.
-__device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  const uint32_t addr = smem_u32(bar);
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 0; !mbar_try_wait(addr, parity); ++it) {
-    if ((it & 63u) == 63u && (globaltimer_ns() - t0 > limit_ns || it >= (1u << 28))) return;
-  }
-}
-
 // Maximum of the 32 values of one chunk (three-input max, 16 instructions).
 __device__ __forceinline__ float chunk_max(const uint32_t* v) {
   float m = fmaxf(__uint_as_float(v[0]), __uint_as_float(v[1]));

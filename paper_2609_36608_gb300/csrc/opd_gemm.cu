@@ -80,14 +80,6 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
 }
 
-__device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
-  const uint32_t addr = smem_u32(bar);
-  const uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 0; !mbar_try_wait(addr, parity); ++it) {
-    if ((it & 63u) == 63u && (globaltimer_ns() - t0 > limit_ns || it >= (1u << 28))) return;
-  }
-}
-
 template <bool A_MN, bool B_MN, bool PAIR>
 __global__ void __launch_bounds__(192, 1)
     k_umma_gemm(const __grid_constant__ CUtensorMap tm_a, const __grid_constant__ CUtensorMap tm_b,
