@@ -449,11 +449,14 @@ def run_gpu(args):
     torch.cuda.synchronize()
     opd_kl.opd_kl_profile_start()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]  # end of each step
     ev0.record()
-    for _ in range(args.steps):
+    for k in range(args.steps):
         step(inputs)
+        marks[k].record()
     ev1.record()
     torch.cuda.synchronize()
+    per_step = [ev0.elapsed_time(marks[0])] + [marks[k - 1].elapsed_time(marks[k]) for k in range(1, args.steps)]
     barrier(world)
     prof = opd_kl.opd_kl_profile_stop()
     if sampler:
@@ -539,7 +542,9 @@ def run_gpu(args):
     clocks = sampler.summary() if sampler else None
     out = {
         "metric": PATH_METRICS[args.path], "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms_step,
+        "ms_per_step_median": float(np.median(per_step)), "ms_per_step_min_max": [min(per_step), max(per_step)],
+        "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded counter-based generator, packed multi-turn layout with masked observations "
                 "and inserted tokens",
