@@ -1,0 +1,99 @@
+"""torch.autograd entry points over the C ABI (argument marshalling only; every step runs
+in libopdkl.so).
+
+OPDReverseKL: per-token reverse KL(student || teacher) of Section 3, Eq. reverse-kl, masked
+to supervised rows; its backward calls opd_kl_backward with the upstream per-token gradient.
+The teacher is frozen (Appendix B.4), so H_t and W_t get no gradient.
+
+OPDSeqMeanKLLoss: the paper's batch loss over the per-token KL (Appendix B.4,
+seq-mean-token-mean), computed with its gradients by one opd_kl_seq_mean_fwd_bwd call in
+the forward; the backward scales those gradients by the upstream scalar.
+
+Gradients come back in the dtype of the tensors they belong to (autograd's rule); the
+library computes them in float32.
+"""
+
+from __future__ import annotations
+
+import torch
+
+from . import opd_kl
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return opd_kl.OPD_DTYPE_BF16
+    if t.dtype == torch.float32:
+        return opd_kl.OPD_DTYPE_F32
+    raise TypeError(f"hidden states and heads must be bfloat16 or float32, not {t.dtype}")
+
+
+def _problem(H_s, H_t, W_s, W_t, temperature):
+    if not (H_s.dtype == H_t.dtype == W_s.dtype == W_t.dtype):
+        raise TypeError("H_s, H_t, W_s and W_t must share one dtype")
+    return opd_kl.make_problem(H_s.shape[0], H_s.shape[1], H_t.shape[1], W_s.shape[0], _dtype_code(H_s),
+                               float(temperature))
+
+
+def _contig(*ts):
+    return [t.contiguous() for t in ts]
+
+
+class OPDReverseKL(torch.autograd.Function):
+    """kl = OPDReverseKL.apply(H_s, H_t, W_s, W_t, mask, temperature) -> [T] float32."""
+
+    @staticmethod
+    def forward(ctx, H_s, H_t, W_s, W_t, mask, temperature=1.0):
+        H_s, H_t, W_s, W_t = _contig(H_s, H_t, W_s, W_t)
+        mask = mask.to(torch.uint8).contiguous()
+        prob = _problem(H_s, H_t, W_s, W_t, temperature)
+        ws = opd_kl.allocate_workspace(prob, H_s.device)
+        T = H_s.shape[0]
+        kl = torch.empty(T, device=H_s.device, dtype=torch.float32)
+        stats = torch.empty(T, 3, device=H_s.device, dtype=torch.float32)
+        opd_kl.opd_kl_forward(prob, H_s, H_t, W_s, W_t, mask, kl, stats, ws)
+        ctx.save_for_backward(H_s, H_t, W_s, W_t, mask, stats)
+        ctx.temperature = float(temperature)
+        ctx.mark_non_differentiable(mask)
+        return kl
+
+    @staticmethod
+    def backward(ctx, grad_kl):
+        H_s, H_t, W_s, W_t, mask, stats = ctx.saved_tensors
+        prob = _problem(H_s, H_t, W_s, W_t, ctx.temperature)
+        ws = opd_kl.allocate_workspace(prob, H_s.device)
+        dH = torch.empty(H_s.shape, device=H_s.device, dtype=torch.float32)
+        dW = torch.empty(W_s.shape, device=W_s.device, dtype=torch.float32)
+        opd_kl.opd_kl_backward(prob, H_s, H_t, W_s, W_t, mask, stats, grad_kl.float().contiguous(), dH, dW, False, ws)
+        return dH.to(H_s.dtype), None, dW.to(W_s.dtype), None, None, None
+
+
+class OPDSeqMeanKLLoss(torch.autograd.Function):
+    """loss = OPDSeqMeanKLLoss.apply(H_s, H_t, W_s, W_t, mask, seg_id, n_ids, temperature, eps)
+    -> scalar float32: L = sum_i w_i KL_i with the paper's seq-mean-token-mean weights."""
+
+    @staticmethod
+    def forward(ctx, H_s, H_t, W_s, W_t, mask, seg_id, n_ids, temperature=1.0, eps=1e-8):
+        H_s, H_t, W_s, W_t = _contig(H_s, H_t, W_s, W_t)
+        mask = mask.to(torch.uint8).contiguous()
+        seg_id = seg_id.to(torch.int32).contiguous()
+        prob = _problem(H_s, H_t, W_s, W_t, temperature)
+        ws = opd_kl.allocate_seq_mean_workspace(prob, int(n_ids), H_s.device)
+        T = H_s.shape[0]
+        dev = H_s.device
+        loss = torch.empty(1, device=dev, dtype=torch.float32)
+        kl = torch.empty(T, device=dev, dtype=torch.float32)
+        stats = torch.empty(T, 3, device=dev, dtype=torch.float32)
+        dH = torch.empty(H_s.shape, device=dev, dtype=torch.float32)
+        dW = torch.empty(W_s.shape, device=dev, dtype=torch.float32)
+        opd_kl.opd_kl_seq_mean_fwd_bwd(prob, H_s, H_t, W_s, W_t, mask, seg_id, int(n_ids), float(eps), loss, kl,
+                                       stats, dH, dW, False, ws)
+        ctx.save_for_backward(dH, dW)
+        ctx.dtypes = (H_s.dtype, W_s.dtype)
+        return loss[0]
+
+    @staticmethod
+    def backward(ctx, grad_loss):
+        dH, dW = ctx.saved_tensors
+        g = grad_loss.float()
+        return (dH * g).to(ctx.dtypes[0]), None, (dW * g).to(ctx.dtypes[1]), None, None, None, None, None, None
