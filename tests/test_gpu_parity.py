@@ -185,6 +185,22 @@ def test_forward_then_backward_matches_fused_call(lib):
     assert _rel(b["dW"], a["dW"].astype(np.float64)) < 1e-5
 
 
+def test_repeated_calls_are_deterministic(lib):
+    """The forward writes each split's partial statistics once and combines them in a fixed
+    order, and dW_s tiles are stored (K = R whole per tile), so KL, stats and dW_s repeat bit for
+    bit. dH_s sums split-K partials by reduce-adds in arrival order: equal to rounding."""
+    w = _small_bf16(T=600, V=3000, seed=29)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    a = _run(lib, w, x, lay.mask, g)
+    b = _run(lib, w, x, lay.mask, g)
+    np.testing.assert_array_equal(a["kl"], b["kl"])
+    np.testing.assert_array_equal(a["stats"], b["stats"])
+    np.testing.assert_array_equal(a["dW"], b["dW"])
+    assert _rel(a["dH"], b["dH"].astype(np.float64)) < 1e-6
+
+
 def test_accumulate_dW_adds(lib):
     w = _small_bf16(T=300, seed=15)
     lay = synth.layout(w)
