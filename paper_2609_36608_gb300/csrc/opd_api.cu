@@ -406,8 +406,11 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumul
   gh.N = (int32_t)c.p.d_s;
   gh.K = (int32_t)c.p.V;
   gh.k_is_R = 0;
-  gh.max_ksplit = env_int("OPD_KL_MAX_KSPLIT", kMaxKSplit);
-  gh.reduce = 1;
+  // deterministic mode: each dH_s tile takes the whole K = V range and is stored, not
+  // summed from split-K partials whose reduce-adds land in any order
+  const bool deterministic = env_flag("OPD_KL_DETERMINISTIC");
+  gh.max_ksplit = deterministic ? 1 : env_int("OPD_KL_MAX_KSPLIT", kMaxKSplit);
+  gh.reduce = deterministic ? 0 : 1;
   gh.pair = gemm_pair_mode();
   gh.work_slot = 2;
   gh.wait_limit_ns = kDefaultWaitLimitNs;

@@ -201,6 +201,18 @@ def test_repeated_calls_are_deterministic(lib):
     assert _rel(a["dH"], b["dH"].astype(np.float64)) < 1e-6
 
 
+def test_deterministic_mode(lib, oracle_mod, monkeypatch):
+    """OPD_KL_DETERMINISTIC=1: dH_s tiles take the whole K range and are stored, so every output
+    repeats bit for bit, and the results still match the oracle."""
+    monkeypatch.setenv("OPD_KL_DETERMINISTIC", "1")
+    w = _small_bf16(T=600, V=3000, seed=30)
+    a, _, x = _full_check(lib, oracle_mod, w)
+    lay = synth.layout(w)
+    b = _run(lib, w, x, lay.mask, synth.uniform_weights(w.seed, w.T))
+    for k in ("kl", "stats", "dH", "dW"):
+        np.testing.assert_array_equal(a[k], b[k])
+
+
 def test_accumulate_dW_adds(lib):
     w = _small_bf16(T=300, seed=15)
     lay = synth.layout(w)
