@@ -91,7 +91,10 @@ typedef struct {
 /* Bytes of device workspace that forward, backward and fwd_bwd need for this
  * problem (an upper bound: it assumes every row may be supervised). Returns 0
  * for an invalid problem. The workspace must be 256-byte aligned. Its largest
- * part is the bf16 dz buffer of T x V elements. */
+ * part is the bf16 dz buffer of T x V elements. To bound it, split a batch into
+ * row chunks: give each chunk its rows' upstream weights (computed once for the
+ * whole batch) and pass accumulate_dW = 1 after the first chunk; the results equal
+ * one call over the whole batch. */
 size_t opd_kl_workspace_size(const opd_problem* problem);
 
 /* Forward (Eq. reverse-kl): per-token KL and the per-row statistics the backward

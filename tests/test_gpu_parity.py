@@ -213,6 +213,29 @@ def test_deterministic_mode(lib, oracle_mod, monkeypatch):
         np.testing.assert_array_equal(a[k], b[k])
 
 
+def test_row_chunks_with_accumulate_equal_one_call(lib):
+    """A batch split into row chunks (per-token upstream weights computed once for the whole
+    batch, one call per chunk, dW_s accumulated after the first) reproduces the single call: the
+    way to bound the workspace (its dz buffer grows as T x V)."""
+    w = _small_bf16(T=900, V=2000, seed=31)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    whole = _run(lib, w, x, lay.mask, g)
+    cuts = [0, 300, 650, 900]
+    dW = torch.zeros(w.V, w.d_s, device="cuda")
+    kl, dH = np.zeros(w.T, np.float32), np.zeros((w.T, w.d_s), np.float32)
+    for i, (a, b) in enumerate(zip(cuts[:-1], cuts[1:])):
+        wc = synth.scaled(w, T=b - a)
+        xc = {"H_s": x["H_s"][a:b], "H_t": x["H_t"][a:b], "W_s": x["W_s"], "W_t": x["W_t"]}
+        out = _run(lib, wc, xc, lay.mask[a:b], g[a:b], accumulate=i > 0, dW_init=dW)
+        dW = torch.from_numpy(out["dW"]).cuda()
+        kl[a:b], dH[a:b] = out["kl"], out["dH"]
+    np.testing.assert_array_equal(kl, whole["kl"])
+    assert _rel(dH, whole["dH"].astype(np.float64)) < 1e-5
+    assert _rel(dW.cpu().numpy(), whole["dW"].astype(np.float64)) < 1e-5
+
+
 def test_accumulate_dW_adds(lib):
     w = _small_bf16(T=300, seed=15)
     lay = synth.layout(w)
