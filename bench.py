@@ -10,8 +10,9 @@ d_t = 4096, V = 151,936, bf16). Metric: supervised response tokens per second.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
 
 Inputs stay resident in HBM for `value`; `e2e` repeats the measurement through
-the same C ABI with the per-step inputs copied from pinned host memory and the
-per-token KL copied back every step. W_s + W_t (1.87 GB) exceed L2 (129 MB), so
+the same C ABI with the per-step inputs copied from pinned host memory (the next
+step's copy overlapping the current step) and the per-token KL copied back every
+step. W_s + W_t (1.87 GB) exceed L2 (129 MB), so
 every step streams the heads from HBM. `--impl reference` times the float64
 CPU oracle on a bounded row sample of the same workload instead.
 """
@@ -629,8 +630,9 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--path", default="kl", choices=sorted(PATH_METRICS),
-                    help="kl: the reverse-KL step (default, the headline); surrogate: the sampled-token "
-                         "dual-clip surrogate; score: teacher token scoring")
+                    help="kl: the reverse-KL step (default, the headline); kl_seqmean: the same step "
+                         "with the paper's batch loss aggregated on the device; surrogate: the "
+                         "sampled-token dual-clip surrogate; score: teacher token scoring")
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
     ap.add_argument("--cpu-rows-1t", type=int, default=4, help="rows of the one-core CPU-oracle sample")
     ap.add_argument("--ref-rows", type=int, default=16, help="rows per step of --impl reference (the oracle splits rows over the host cores)")
