@@ -307,6 +307,7 @@ def path_setup(path, w, lay, x, dev, opd_kl):
         def step(i):
             opd_kl.opd_kl_fwd_bwd(prob, i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["grad"], kl, stats, dH,
                                   dW, False, ws)
+        step.outputs = {"kl": kl, "dH": dH}
         executed, algorithmic = step_flops(w, R)
         return inputs, step, kl, ws, executed, algorithmic
     if path == "kl_seqmean":
@@ -321,6 +322,7 @@ def path_setup(path, w, lay, x, dev, opd_kl):
         def step(i):
             opd_kl.opd_kl_seq_mean_fwd_bwd(prob, i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["seg_id"],
                                            n_ids, 1e-8, loss, kl, stats, dH, dW, False, ws)
+        step.outputs = {"kl": kl, "dH": dH}
         executed, algorithmic = step_flops(w, R)
         return inputs, step, loss, ws, executed, algorithmic
     tokens = torch.from_numpy(synth.token_ids(w.seed, w.T, w.V)).to(dev)
@@ -332,6 +334,7 @@ def path_setup(path, w, lay, x, dev, opd_kl):
 
         def step(i):
             opd_kl.opd_score_tokens(prob, i["H_t"], x["W_t"], i["tokens"], i["mask"], lse, logp, ws)
+        step.outputs = {"lse": lse, "logp": logp}
         fl = 2.0 * R * w.V * w.d_t
         return inputs, step, logp, ws, fl, fl
     # surrogate: synthetic teacher and behaviour log-probabilities (the teacher enters only there)
@@ -355,6 +358,8 @@ def path_setup(path, w, lay, x, dev, opd_kl):
         opd_kl.opd_surrogate_fwd_bwd(prob, i["H_s"], x["W_s"], i["tokens"], i["logp_old"], i["logp_teacher"],
                                      i["mask"], dev_w, loss, logp, dH, dW, False, ws)
         opd_kl.opd_seq_mean_token_mean_device(i["seg_id"], i["mask"], n_ids, 1e-8, loss, None, total, seq_ws)
+    step.outputs = {"loss": loss, "logp": logp, "dH": dH}
+    step.oracle_inputs = {"logp_old": logp_old, "logp_teacher": logp_teacher}
     return inputs, step, total, ws, 8.0 * R * w.V * w.d_s, 6.0 * R * w.V * w.d_s
 
 
@@ -369,9 +374,10 @@ def path_kernel_flops(path, name, w, R):
     return None
 
 
-def path_cpu_baseline(path, w, lay, x, args):
+def path_cpu_baseline(path, w, lay, x, args, step=None):
     """The oracle, as it stands, on a bounded row sample of the same workload: on every host
-    core, and on one core for a smaller sample."""
+    core, and on one core for a smaller sample. With the step's GPU outputs, also the parity of
+    those rows (the bench's own launch configuration against the oracle)."""
     import oracle
     oracle.build()
     threads = os.cpu_count() or 1
@@ -381,8 +387,8 @@ def path_cpu_baseline(path, w, lay, x, args):
         g = np.where(lay.mask != 0, opd_seq_weights(lay), 0.0)
 
         def run(rs, n):
-            oracle.opd_kl(host["H_s"], host["H_t"], host["W_s"], host["W_t"], lay.mask, g, w.tau, rows=rs,
-                          want_dH=True, want_dW=True, n_threads=n)
+            return oracle.opd_kl(host["H_s"], host["H_t"], host["W_s"], host["W_t"], lay.mask, g, w.tau, rows=rs,
+                                 want_dH=True, want_dW=True, n_threads=n)
         what = "float64 logits, KL, dH_s rows and their dW_s contribution"
     else:
         tokens = synth.token_ids(w.seed, w.T, w.V)
@@ -390,28 +396,63 @@ def path_cpu_baseline(path, w, lay, x, args):
             H, W = synth.host_values(x["H_t"]), synth.host_values(x["W_t"])
 
             def run(rs, n):
-                oracle.score(H, W, tokens, w.tau, rows=rs, n_threads=n)
+                return oracle.score(H, W, tokens, w.tau, rows=rs, n_threads=n)
             what = "float64 teacher log-partition and token log-probabilities"
         else:
-            H, W, T = synth.host_values(x["H_s"]), synth.host_values(x["W_s"]), w.T
+            # the GPU step's own behaviour and teacher log-probabilities and seq-mean weights
+            H, W = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+            extra = getattr(step, "oracle_inputs", {})
+            lo = extra["logp_old"].double().cpu().numpy() if extra else np.full(w.T, -7.0)
+            lt = extra["logp_teacher"].double().cpu().numpy() if extra else np.full(w.T, -7.0)
+            sw = opd_seq_weights(lay)
 
             def run(rs, n):
-                oracle.surrogate(H, W, tokens, np.full(T, -7.0), np.full(T, -7.0), lay.mask, np.ones(T), w.tau,
-                                 rows=rs, n_threads=n)
+                return oracle.surrogate(H, W, tokens, lo, lt, lay.mask, sw, w.tau, rows=rs, n_threads=n)
             what = "float64 student logits, dual-clip loss, dH_s rows and their dW_s contribution"
 
     def timed(rs, n):
         t0 = time.perf_counter()
-        run(rs, n)
-        return time.perf_counter() - t0
+        res = run(rs, n)
+        return time.perf_counter() - t0, res
 
-    dt = timed(rows, threads)
+    dt, ref = timed(rows, threads)
     rows1 = rows[:max(1, min(len(rows), args.cpu_rows_1t))]
-    dt1 = timed(rows1, 1)
-    return {"value": len(rows) / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"{len(rows)} supervised rows of {w.name}: {what} ({dt:.1f} s)",
-            "value_1_thread": len(rows1) / dt1,
-            "sample_1_thread": f"the first {len(rows1)} of those rows on one core ({dt1:.1f} s)"}
+    dt1, _ = timed(rows1, 1)
+    out = {"value": len(rows) / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+           "sample": f"{len(rows)} supervised rows of {w.name}: {what} ({dt:.1f} s)",
+           "value_1_thread": len(rows1) / dt1,
+           "sample_1_thread": f"the first {len(rows1)} of those rows on one core ({dt1:.1f} s)"}
+    return out, sampled_parity(path, rows, ref, getattr(step, "outputs", None))
+
+
+def sampled_parity(path, rows, ref, outputs):
+    """Errors of the timed GPU step's outputs on the oracle's sampled rows, against the
+    parity bounds (KL and per-token loss: 1e-4 + 2e-3 |x|; dH_s: 1e-2 relative Frobenius;
+    lse and logp: 1e-4 + 1e-4 |x|)."""
+    if not outputs:
+        return None
+    sel = torch.as_tensor(rows, device=next(iter(outputs.values())).device)
+    pick = {k: v.index_select(0, sel).double().cpu().numpy() for k, v in outputs.items()}
+    if path in ("kl", "kl_seqmean"):
+        err = np.abs(pick["kl"] - ref.kl)
+        rel = float(np.linalg.norm(pick["dH"] - ref.dH_s) / max(np.linalg.norm(ref.dH_s), 1e-300))
+        return {"rows": len(rows), "kl_max_abs_err": float(err.max()),
+                "kl_within_bound": bool((err <= 1e-4 + 2e-3 * np.abs(ref.kl)).all()),
+                "dH_rel_fro_err": rel, "dH_within_bound": rel <= 1e-2}
+    if path == "surrogate":
+        e1, e2 = np.abs(pick["logp"] - ref.logp_s), np.abs(pick["loss"] - ref.loss)
+        rel = float(np.linalg.norm(pick["dH"] - ref.dH_s) / max(np.linalg.norm(ref.dH_s), 1e-300))
+        return {"rows": len(rows), "logp_max_abs_err": float(e1.max()), "loss_max_abs_err": float(e2.max()),
+                "dH_rel_fro_err": rel,
+                "within_bound": bool((e1 <= 1e-4 + 1e-4 * np.abs(ref.logp_s)).all()
+                                     and (e2 <= 1e-4 + 2e-3 * np.abs(ref.loss)).all() and rel <= 1e-2)}
+    if path == "score":
+        lse_ref, lp_ref = ref
+        e1, e2 = np.abs(pick["lse"] - lse_ref), np.abs(pick["logp"] - lp_ref)
+        return {"rows": len(rows), "lse_max_abs_err": float(e1.max()), "logp_max_abs_err": float(e2.max()),
+                "within_bound": bool((e1 <= 1e-4 + 1e-4 * np.abs(lse_ref)).all()
+                                     and (e2 <= 1e-4 + 1e-4 * np.abs(lp_ref)).all())}
+    return None
 
 
 def opd_seq_weights(lay):
@@ -536,9 +577,9 @@ def run_gpu(args):
                     "frac_of_burst": achieved / peaks["bf16_tflops"],
                     "algorithmic_flops_per_launch": per_launch}
 
-    cpu = None
+    cpu, parity = None, None
     if world == 1 and not args.no_cpu_baseline:
-        cpu = path_cpu_baseline(args.path, w, lay, x, args)
+        cpu, parity = path_cpu_baseline(args.path, w, lay, x, args, step)
 
     clocks = sampler.summary() if sampler else None
     out = {
@@ -557,6 +598,7 @@ def run_gpu(args):
         "pct_bf16_peak_executed": 100.0 * executed / (ms_step / 1000.0) / 1e12 / peaks["bf16_tflops"],
         "roofline": roofline,
         "cpu_baseline": cpu,
+        "parity_sampled_rows": parity,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
         "clocks": clocks,
