@@ -131,6 +131,19 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(self.rows), "power_w_max": max(pw) if pw else None}
 
 
+def choose_peak(clocks, peaks, peak_src):
+    """The bf16 denominator for a kernel timed inside the benchmark's step: the sustained
+    figure when the step ran under the power limiter (sw_power_cap seen, or the median SM
+    clock below 95% of its maximum), else the burst figure. Without a clock record the
+    burst figure (the larger one) is used. Returns (peak, description)."""
+    capped = bool(clocks) and (
+        "sw_power_cap" in (clocks.get("reasons") or [])
+        or (clocks.get("sm_mhz") and clocks.get("sm_max_mhz") and clocks["sm_mhz"] < 0.95 * clocks["sm_max_mhz"]))
+    if capped:
+        return peaks["bf16_tflops_sustained"], f"bf16_tflops_sustained of {peak_src} (the step ran power-capped)"
+    return peaks["bf16_tflops"], f"bf16_tflops (burst) of {peak_src} (the step ran at full clock)"
+
+
 # ------------------------------------------------------------------ distributed
 
 def dist_env():
@@ -559,6 +572,7 @@ def run_gpu(args):
         return 0
 
     peaks, peak_src = load_peaks()
+    clocks = sampler.summary() if sampler else None
     kernels = {}
     total_k = sum(v[1] for v in prof.values()) or 1.0
     for name, (n, tot) in sorted(prof.items(), key=lambda kv: -kv[1][1]):
@@ -569,19 +583,18 @@ def run_gpu(args):
     if dom:
         per_launch = path_kernel_flops(args.path, dom, w, R)
         achieved = per_launch / (kernels[dom]["ms_per_launch"] / 1000.0) / 1e12
-        peak = peaks["bf16_tflops_sustained"]
+        peak, peak_desc = choose_peak(clocks, peaks, peak_src)
         traffic = recorded_traffic(dom, w.name, args.path)
         roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak, "traffic": traffic,
-                    "peak_source": f"bf16_tflops_sustained of {peak_src}",
+                    "frac": achieved / peak, "traffic": traffic, "peak_source": peak_desc,
                     "frac_of_burst": achieved / peaks["bf16_tflops"],
+                    "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
                     "algorithmic_flops_per_launch": per_launch}
 
     cpu, parity = None, None
     if world == 1 and not args.no_cpu_baseline:
         cpu, parity = path_cpu_baseline(args.path, w, lay, x, args, step)
 
-    clocks = sampler.summary() if sampler else None
     out = {
         "metric": PATH_METRICS[args.path], "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step,
