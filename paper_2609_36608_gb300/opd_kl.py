@@ -97,16 +97,65 @@ def make_problem(T: int, d_s: int, d_t: int, V: int, dtype: int = OPD_DTYPE_BF16
     return opd_problem(int(T), int(d_s), int(d_t), int(V), int(dtype), float(temperature))
 
 
-def _ptr(t: Optional[torch.Tensor]):
-    if t is None:
-        return None
-    if not isinstance(t, torch.Tensor):
-        raise TypeError("expected a torch.Tensor")
-    if not t.is_cuda:
-        raise ValueError("device buffers must be CUDA tensors")
-    if not t.is_contiguous():
-        raise ValueError("buffers must be contiguous")
-    return ctypes.c_void_p(t.data_ptr()) if t.numel() > 0 else None
+_F32 = (torch.float32,)
+_I32 = (torch.int32,)
+_BYTE = (torch.uint8, torch.bool)  # one byte per row, nonzero = supervised
+
+
+class _Buffers:
+    """Device pointers of the buffers one call reads or writes.
+
+    The library sees only the pointers, so every buffer is checked here against what the
+    call will touch: a contiguous tensor of the element type the C signature documents,
+    holding at least `numel` elements; then, once every buffer has passed that, a CUDA
+    tensor on the current device. A wrong buffer raises before any launch instead of
+    reaching a kernel. None passes through as NULL (the C entry points reject a NULL
+    they need)."""
+
+    def __init__(self):
+        self.seen = []
+
+    def __call__(self, t: Optional[torch.Tensor], name: str, dtypes=None, numel: int = 0):
+        if t is None:
+            return None
+        if not isinstance(t, torch.Tensor):
+            raise TypeError(f"{name}: expected a torch.Tensor")
+        if dtypes is not None and t.dtype not in dtypes:
+            raise TypeError(f"{name}: dtype {t.dtype}, expected {' or '.join(str(d) for d in dtypes)}")
+        if not t.is_contiguous():
+            raise ValueError(f"{name}: buffers must be contiguous")
+        if t.numel() < numel:
+            raise ValueError(f"{name} holds {t.numel()} elements; the problem needs {numel}")
+        self.seen.append((name, t))
+        return ctypes.c_void_p(t.data_ptr()) if t.numel() > 0 else None
+
+    def on_device(self) -> None:
+        for name, t in self.seen:
+            if not t.is_cuda:
+                raise ValueError(f"{name}: device buffers must be CUDA tensors")
+            if t.device.index != torch.cuda.current_device():
+                raise ValueError(f"{name} is on {t.device}, but the current device is "
+                                 f"cuda:{torch.cuda.current_device()}")
+
+
+def _nbytes(t: Optional[torch.Tensor]) -> int:
+    return 0 if t is None else t.numel() * t.element_size()
+
+
+def _inputs(problem) -> tuple:
+    return (torch.bfloat16,) if problem.dtype == OPD_DTYPE_BF16 else (torch.float32,)
+
+
+def _kl_inputs(b: _Buffers, problem, H_s, H_t, W_s, W_t, mask) -> list:
+    T, ds, dt, V, x = problem.T, problem.d_s, problem.d_t, problem.V, _inputs(problem)
+    return [b(H_s, "H_s", x, T * ds), b(H_t, "H_t", x, T * dt), b(W_s, "W_s", x, V * ds), b(W_t, "W_t", x, V * dt),
+            b(mask, "mask", _BYTE, T)]
+
+
+def _call(name: str, b: _Buffers, args: list, stream) -> int:
+    """Checks the buffers' device, then calls the entry point with the stream appended."""
+    b.on_device()
+    return int(getattr(_lib, name)(*args, _stream(stream)))
 
 
 def _stream(stream) -> ctypes.c_void_p:
@@ -134,33 +183,40 @@ def allocate_workspace(problem: opd_problem, device="cuda") -> torch.Tensor:
 
 
 def opd_kl_forward(problem, H_s, H_t, W_s, W_t, mask, kl_out, stats, workspace, stream=None) -> None:
-    _check(_lib.opd_kl_forward(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
-                               _ptr(kl_out), _ptr(stats), _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_kl_forward")
+    T, b = problem.T, _Buffers()
+    args = [ctypes.byref(problem), *_kl_inputs(b, problem, H_s, H_t, W_s, W_t, mask),
+            b(kl_out, "kl_out", _F32, T), b(stats, "stats", _F32, 3 * T),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_kl_forward", b, args, stream), "opd_kl_forward")
 
 
 def opd_kl_forward_noalloc(problem, H_s, H_t, W_s, W_t, mask, kl_out, stats, stream=None) -> None:
     """opd_kl_forward without a workspace, for callers that may not allocate device memory
     (T <= OPD_KL_NOALLOC_MAX_ROWS, bf16; scratch is a fixed array inside the library)."""
-    _check(_lib.opd_kl_forward_noalloc(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t),
-                                       _ptr(mask), _ptr(kl_out), _ptr(stats), _stream(stream)),
-           "opd_kl_forward_noalloc")
+    T, b = problem.T, _Buffers()
+    args = [ctypes.byref(problem), *_kl_inputs(b, problem, H_s, H_t, W_s, W_t, mask),
+            b(kl_out, "kl_out", _F32, T), b(stats, "stats", _F32, 3 * T)]
+    _check(_call("opd_kl_forward_noalloc", b, args, stream), "opd_kl_forward_noalloc")
 
 
 def opd_kl_backward(problem, H_s, H_t, W_s, W_t, mask, stats, grad_kl, dH_s, dW_s, accumulate_dW: bool,
                     workspace, stream=None) -> None:
-    _check(_lib.opd_kl_backward(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
-                                _ptr(stats), _ptr(grad_kl), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
-                                _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_kl_backward")
+    T, ds, V, b = problem.T, problem.d_s, problem.V, _Buffers()
+    args = [ctypes.byref(problem), *_kl_inputs(b, problem, H_s, H_t, W_s, W_t, mask),
+            b(stats, "stats", _F32, 3 * T), b(grad_kl, "grad_kl", _F32, T), b(dH_s, "dH_s", _F32, T * ds),
+            b(dW_s, "dW_s", _F32, V * ds), int(bool(accumulate_dW)),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_kl_backward", b, args, stream), "opd_kl_backward")
 
 
 def opd_kl_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, grad_kl, kl_out, stats, dH_s, dW_s, accumulate_dW: bool,
                    workspace, stream=None) -> None:
-    _check(_lib.opd_kl_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t), _ptr(mask),
-                               _ptr(grad_kl), _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s),
-                               int(bool(accumulate_dW)), _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_kl_fwd_bwd")
+    T, ds, V, b = problem.T, problem.d_s, problem.V, _Buffers()
+    args = [ctypes.byref(problem), *_kl_inputs(b, problem, H_s, H_t, W_s, W_t, mask),
+            b(grad_kl, "grad_kl", _F32, T), b(kl_out, "kl_out", _F32, T), b(stats, "stats", _F32, 3 * T),
+            b(dH_s, "dH_s", _F32, T * ds), b(dW_s, "dW_s", _F32, V * ds), int(bool(accumulate_dW)),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_kl_fwd_bwd", b, args, stream), "opd_kl_fwd_bwd")
 
 
 def opd_kl_seq_mean_workspace_size(problem, n_ids: int) -> int:
@@ -178,29 +234,35 @@ def opd_kl_seq_mean_fwd_bwd(problem, H_s, H_t, W_s, W_t, mask, seg_id, n_ids: in
                             stats, dH_s, dW_s, accumulate_dW: bool, workspace, stream=None) -> None:
     """The paper's batch loss over the per-token KL (seq-mean-token-mean weights on the device, L summed
     in the combine pass) and its gradients, in one call."""
-    _check(_lib.opd_kl_seq_mean_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(H_t), _ptr(W_s), _ptr(W_t),
-                                        _ptr(mask), _ptr(seg_id), int(n_ids), float(eps), _ptr(loss_out),
-                                        _ptr(kl_out), _ptr(stats), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
-                                        _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_kl_seq_mean_fwd_bwd")
+    T, ds, V, b = problem.T, problem.d_s, problem.V, _Buffers()
+    args = [ctypes.byref(problem), *_kl_inputs(b, problem, H_s, H_t, W_s, W_t, mask),
+            b(seg_id, "seg_id", _I32, T), int(n_ids), float(eps), b(loss_out, "loss_out", _F32, 1),
+            b(kl_out, "kl_out", _F32, T), b(stats, "stats", _F32, 3 * T), b(dH_s, "dH_s", _F32, T * ds),
+            b(dW_s, "dW_s", _F32, V * ds), int(bool(accumulate_dW)),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_kl_seq_mean_fwd_bwd", b, args, stream), "opd_kl_seq_mean_fwd_bwd")
 
 
 def opd_score_tokens(problem, H, W, tokens, mask, lse_out, logp_out, workspace, stream=None) -> None:
     """Log-partition and log-probability of the given tokens under one head (d = problem.d_s)."""
-    _check(_lib.opd_score_tokens(ctypes.byref(problem), _ptr(H), _ptr(W), _ptr(tokens), _ptr(mask), _ptr(lse_out),
-                                 _ptr(logp_out), _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_score_tokens")
+    T, d, V, x, b = problem.T, problem.d_s, problem.V, _inputs(problem), _Buffers()
+    args = [ctypes.byref(problem), b(H, "H", x, T * d), b(W, "W", x, V * d), b(tokens, "tokens", _I32, T),
+            b(mask, "mask", _BYTE, T), b(lse_out, "lse_out", _F32, T), b(logp_out, "logp_out", _F32, T),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_score_tokens", b, args, stream), "opd_score_tokens")
 
 
 def opd_surrogate_fwd_bwd(problem, H_s, W_s, tokens, logp_old, logp_teacher, mask, weights, loss_out, logp_out,
                           dH_s, dW_s, accumulate_dW: bool, workspace, params=None, stream=None) -> None:
     """Sampled-token dual-clip surrogate, forward and backward (student side)."""
+    T, d, V, x, b = problem.T, problem.d_s, problem.V, _inputs(problem), _Buffers()
     pp = ctypes.byref(params) if params is not None else None
-    _check(_lib.opd_surrogate_fwd_bwd(ctypes.byref(problem), _ptr(H_s), _ptr(W_s), _ptr(tokens), _ptr(logp_old),
-                                      _ptr(logp_teacher), _ptr(mask), _ptr(weights), pp, _ptr(loss_out),
-                                      _ptr(logp_out), _ptr(dH_s), _ptr(dW_s), int(bool(accumulate_dW)),
-                                      _ptr(workspace), workspace.numel(), _stream(stream)),
-           "opd_surrogate_fwd_bwd")
+    args = [ctypes.byref(problem), b(H_s, "H_s", x, T * d), b(W_s, "W_s", x, V * d), b(tokens, "tokens", _I32, T),
+            b(logp_old, "logp_old", _F32, T), b(logp_teacher, "logp_teacher", _F32, T), b(mask, "mask", _BYTE, T),
+            b(weights, "weights", _F32, T), pp, b(loss_out, "loss_out", _F32, T), b(logp_out, "logp_out", _F32, T),
+            b(dH_s, "dH_s", _F32, T * d), b(dW_s, "dW_s", _F32, V * d), int(bool(accumulate_dW)),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_surrogate_fwd_bwd", b, args, stream), "opd_surrogate_fwd_bwd")
 
 
 def opd_seq_mean_token_mean_weights(seg_id, mask, eps: float = 1e-8) -> np.ndarray:
@@ -224,19 +286,23 @@ def opd_seq_mean_token_mean_device(seg_id, mask, n_ids: int, eps: float = 1e-8, 
     if workspace is None:
         workspace = torch.empty(opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8,
                                 device=seg_id.device)
-    _check(_lib.opd_seq_mean_token_mean_device(_ptr(seg_id), _ptr(mask), seg_id.numel(), int(n_ids), float(eps),
-                                               _ptr(loss_in), _ptr(w_out), _ptr(loss_out), _ptr(workspace),
-                                               workspace.numel(), _stream(stream)),
-           "opd_seq_mean_token_mean_device")
+    T, b = seg_id.numel(), _Buffers()
+    args = [b(seg_id, "seg_id", _I32, T), b(mask, "mask", _BYTE, T), T, int(n_ids), float(eps),
+            b(loss_in, "loss_in", _F32, T), b(w_out, "w_out", _F32, T), b(loss_out, "loss_out", _F32, 1),
+            b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_seq_mean_token_mean_device", b, args, stream), "opd_seq_mean_token_mean_device")
     return workspace
 
 
 def opd_kl_get_status(workspace, stream=None) -> int:
-    return int(_lib.opd_kl_get_status(_ptr(workspace), workspace.numel(), _stream(stream)))
+    b = _Buffers()
+    return _call("opd_kl_get_status", b, [b(workspace, "workspace"), _nbytes(workspace)], stream)
 
 
 def opd_kl_selftest_timeout(workspace, limit_ns: int, stream=None) -> int:
-    return int(_lib.opd_kl_selftest_timeout(_ptr(workspace), workspace.numel(), int(limit_ns), _stream(stream)))
+    b = _Buffers()
+    return _call("opd_kl_selftest_timeout", b, [b(workspace, "workspace"), _nbytes(workspace), int(limit_ns)],
+                 stream)
 
 
 def opd_kl_profile_start() -> None:

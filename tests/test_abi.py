@@ -125,3 +125,50 @@ def test_kl_seq_mean_arguments(lib):
     small = [ctypes.byref(p), fake, fake, fake, fake, fake, fake, ctypes.c_int64(10), ctypes.c_float(1e-8), fake,
              fake, fake, fake, fake, 0, fake, ctypes.c_size_t(base), None]
     assert lib.call_raw("opd_kl_seq_mean_fwd_bwd", *small) == lib.OPD_ERR_INVALID_ARG  # KL workspace only
+
+
+def test_binding_checks_every_buffer_before_the_call(lib):
+    """The C entry points see bare pointers, so the Python binding checks each buffer's
+    element type, contiguity and size against the problem before calling. The checks run
+    before the CUDA-device check, so host tensors exercise them here."""
+    import torch
+    T, d_s, d_t, V = 8, 16, 24, 40
+    prob = lib.make_problem(T, d_s, d_t, V, lib.OPD_DTYPE_BF16, 1.0)
+    bf = lambda *s: torch.zeros(*s, dtype=torch.bfloat16)
+    f32 = lambda *s: torch.zeros(*s, dtype=torch.float32)
+    mask = torch.ones(T, dtype=torch.uint8)
+    ws = torch.zeros(64, dtype=torch.uint8)
+    good = dict(H_s=bf(T, d_s), H_t=bf(T, d_t), W_s=bf(V, d_s), W_t=bf(V, d_t), mask=mask, kl_out=f32(T),
+                stats=f32(T, 3), workspace=ws)
+
+    def call(**over):
+        a = dict(good, **over)
+        lib.opd_kl_forward(prob, a["H_s"], a["H_t"], a["W_s"], a["W_t"], a["mask"], a["kl_out"], a["stats"],
+                           a["workspace"])
+
+    with pytest.raises(TypeError, match="H_s: dtype torch.float32"):
+        call(H_s=f32(T, d_s))
+    with pytest.raises(ValueError, match="W_t holds"):
+        call(W_t=bf(V - 1, d_t))
+    with pytest.raises(ValueError, match="stats holds"):
+        call(stats=f32(T, 2))
+    with pytest.raises(ValueError, match="H_t: buffers must be contiguous"):
+        call(H_t=bf(d_t, T).t())
+    with pytest.raises(TypeError, match="mask: dtype torch.int64"):
+        call(mask=torch.ones(T, dtype=torch.int64))
+    with pytest.raises(ValueError, match="must be CUDA tensors"):
+        call()  # every size and type right: only the device is wrong
+    with pytest.raises(ValueError, match="must be CUDA tensors"):
+        call(mask=torch.ones(T, dtype=torch.bool))  # one byte per row, accepted
+    g = f32(T)
+    with pytest.raises(ValueError, match="dW_s holds"):
+        lib.opd_kl_fwd_bwd(prob, good["H_s"], good["H_t"], good["W_s"], good["W_t"], mask, g, f32(T), f32(T, 3),
+                           f32(T, d_s), f32(V, d_s - 1), False, ws)
+    with pytest.raises(TypeError, match="tokens: dtype torch.int64"):
+        lib.opd_score_tokens(prob, good["H_s"], good["W_s"], torch.zeros(T, dtype=torch.int64), mask, f32(T),
+                             f32(T), ws)
+    with pytest.raises(TypeError, match="seg_id: dtype torch.int64"):
+        lib.opd_seq_mean_token_mean_device(torch.zeros(T, dtype=torch.int64), mask, 1, 1e-8, None, f32(T), None, ws)
+    f32p = lib.make_problem(T, d_s, d_t, V, lib.OPD_DTYPE_F32, 1.0)
+    with pytest.raises(TypeError, match="H_s: dtype torch.bfloat16"):
+        lib.opd_kl_forward(f32p, good["H_s"], f32(T, d_t), f32(V, d_s), f32(V, d_t), mask, f32(T), f32(T, 3), ws)
