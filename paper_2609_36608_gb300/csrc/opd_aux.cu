@@ -66,25 +66,37 @@ __global__ void __launch_bounds__(kCompactThreads)
   }
 }
 
-// Row gather in 16-byte vectors; rows in [R, R_pad) become zero.
-__global__ void k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict__ Ht, int32_t vs, int32_t vt,
-                          const int32_t* __restrict__ idx, const Ctrl* __restrict__ ctrl, uint4* __restrict__ Hs_g,
-                          uint4* __restrict__ Ht_g) {
+// Row gather in 16-byte vectors; rows in [R, R_pad) become zero. One block per
+// gathered row at a time (no per-element division); each thread loads up to
+// kGatherVec vectors of the row (H_s part, then H_t part) before storing them.
+constexpr int kGatherVec = 4;
+
+__global__ void __launch_bounds__(256) k_gather2(const uint4* __restrict__ Hs, const uint4* __restrict__ Ht,
+                                                 int32_t vs, int32_t vt, const int32_t* __restrict__ idx,
+                                                 const Ctrl* __restrict__ ctrl, uint4* __restrict__ Hs_g,
+                                                 uint4* __restrict__ Ht_g) {
   const int R = ctrl->R;
   const int R_pad = (R + kRowPad - 1) / kRowPad * kRowPad;
   const int per_row = vs + vt;
-  const long total = (long)R_pad * per_row;
-  for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x) {
-    const int r = (int)(e / per_row);
-    const int v = (int)(e - (long)r * per_row);
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (v < vs) {
-      if (r < R) val = Hs[(long)idx[r] * vs + v];
-      Hs_g[(long)r * vs + v] = val;
-    } else {
-      const int v2 = v - vs;
-      if (r < R) val = Ht[(long)idx[r] * vt + v2];
-      Ht_g[(long)r * vt + v2] = val;
+  for (int r = blockIdx.x; r < R_pad; r += gridDim.x) {
+    const bool live = r < R;
+    const long src = live ? (long)idx[r] : 0;
+    for (int v0 = 0; v0 < per_row; v0 += kGatherVec * blockDim.x) {
+      uint4 x[kGatherVec];
+#pragma unroll
+      for (int k = 0; k < kGatherVec; ++k) {
+        const int v = v0 + k * blockDim.x + threadIdx.x;
+        x[k] = make_uint4(0u, 0u, 0u, 0u);
+        if (live && v < per_row) x[k] = v < vs ? Hs[src * vs + v] : Ht[src * vt + (v - vs)];
+      }
+#pragma unroll
+      for (int k = 0; k < kGatherVec; ++k) {
+        const int v = v0 + k * blockDim.x + threadIdx.x;
+        if (v < vs)
+          Hs_g[(long)r * vs + v] = x[k];
+        else if (v < per_row)
+          Ht_g[(long)r * vt + (v - vs)] = x[k];
+      }
     }
   }
 }
@@ -176,14 +188,30 @@ __global__ void k_zero_rows(float4* __restrict__ buf, int32_t vec_per_row, const
     buf[e] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-__global__ void k_scatter_rows(const float4* __restrict__ src, int32_t vec_per_row, const int32_t* __restrict__ pos,
-                               int32_t T, float4* __restrict__ dst) {
-  const long total = (long)T * vec_per_row;
-  for (long e = blockIdx.x * (long)blockDim.x + threadIdx.x; e < total; e += (long)gridDim.x * blockDim.x) {
-    const int i = (int)(e / vec_per_row);
-    const int v = (int)(e - (long)i * vec_per_row);
+// One block per token row at a time (no per-element division); each thread moves
+// up to kScatterVec 16-byte vectors of the row, all loads issued before the stores.
+constexpr int kScatterVec = 4;
+
+__global__ void __launch_bounds__(256) k_scatter_rows(const float4* __restrict__ src, int32_t vec_per_row,
+                                                      const int32_t* __restrict__ pos, int32_t T,
+                                                      float4* __restrict__ dst) {
+  for (int i = blockIdx.x; i < T; i += gridDim.x) {
     const int r = pos[i];
-    dst[e] = r >= 0 ? src[(long)r * vec_per_row + v] : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4* s = src + (long)(r >= 0 ? r : 0) * vec_per_row;
+    float4* d = dst + (long)i * vec_per_row;
+    for (int v0 = 0; v0 < vec_per_row; v0 += kScatterVec * blockDim.x) {
+      float4 x[kScatterVec];
+#pragma unroll
+      for (int k = 0; k < kScatterVec; ++k) {
+        const int v = v0 + k * blockDim.x + threadIdx.x;
+        x[k] = (r >= 0 && v < vec_per_row) ? s[v] : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int k = 0; k < kScatterVec; ++k) {
+        const int v = v0 + k * blockDim.x + threadIdx.x;
+        if (v < vec_per_row) d[v] = x[k];
+      }
+    }
   }
 }
 
@@ -220,7 +248,9 @@ cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t
 cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, int32_t d_t, const int32_t* idx,
                                const Ctrl* ctrl, void* Hs_g, void* Ht_g, int32_t T_pad, int n_sm, cudaStream_t s) {
   const int vs = d_s / 8, vt = d_t / 8;  // 8 bf16 per 16-byte vector
-  k_gather2<<<grid_for((long)T_pad * (vs + vt), n_sm, 256), 256, 0, s>>>(
+  // rows are walked by blocks; R is known only on the device, so the grid covers T_pad rows
+  const long blocks = (long)T_pad < (long)n_sm * 8 ? (long)T_pad : (long)n_sm * 8;
+  k_gather2<<<(int)(blocks < 1 ? 1 : blocks), 256, 0, s>>>(
       static_cast<const uint4*>(H_s), static_cast<const uint4*>(H_t), vs, vt, idx, ctrl,
       static_cast<uint4*>(Hs_g), static_cast<uint4*>(Ht_g));
   return cudaGetLastError();
@@ -248,8 +278,13 @@ cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t
 
 cudaError_t launch_scatter_rows(const float* src_g, int32_t cols, const int32_t* pos, int32_t T, float* dst,
                                 int n_sm, cudaStream_t s) {
-  k_scatter_rows<<<grid_for((long)T * cols / 4, n_sm, 256), 256, 0, s>>>(
-      reinterpret_cast<const float4*>(src_g), cols / 4, pos, T, reinterpret_cast<float4*>(dst));
+  // blocks of 128 threads when a row has at most 512 vectors (d_s <= 2048), so each thread
+  // keeps four vectors in flight; 8 blocks per SM, at most one per row
+  const int vpr = cols / 4;
+  const int threads = vpr <= 512 ? 128 : 256;
+  const long blocks = T < (long)n_sm * 8 ? T : (long)n_sm * 8;
+  k_scatter_rows<<<(int)(blocks < 1 ? 1 : blocks), threads, 0, s>>>(
+      reinterpret_cast<const float4*>(src_g), vpr, pos, T, reinterpret_cast<float4*>(dst));
   return cudaGetLastError();
 }
 
