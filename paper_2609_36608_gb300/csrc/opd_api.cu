@@ -330,6 +330,7 @@ FusedParams fused_params(const Call& c) {
   fp.rowc = reinterpret_cast<const float4*>(c.ws + c.L.rowc);
   fp.mode = fused_tile_mode();
   fp.max_vsplit = kMaxVSplit;
+  fp.half_tile = env_int("OPD_KL_HALF_TILE", 1) != 0 ? 1 : 0;
   return fp;
 }
 

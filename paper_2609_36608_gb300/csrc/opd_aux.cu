@@ -63,6 +63,7 @@ __global__ void __launch_bounds__(kCompactThreads)
   if (tid == kCompactThreads - 1) {
     ctrl->R = warp_tot[31];
     ctrl->n_vsplit = 0;
+    ctrl->half_tile = 0;
   }
 }
 
@@ -124,6 +125,7 @@ __global__ void k_combine(const float* __restrict__ part, const int32_t* __restr
                           const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
                           float* __restrict__ stats, const float* __restrict__ weights, double* loss_acc) {
   const int n_vs = ctrl->n_vsplit;
+  const int h0 = ctrl->half_tile - 1;  // first row of a half-height tile, or -1
   const size_t plane = (size_t)T_pad;
   const int lane = threadIdx.x & 31;
   const int warps = (gridDim.x * blockDim.x) >> 5;
@@ -133,9 +135,14 @@ __global__ void k_combine(const float* __restrict__ part, const int32_t* __restr
     float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
     if (r >= 0 && n_vs > 0) {
       float ms = -CUDART_INF_F, ss = 0.f, as = 0.f, mt = -CUDART_INF_F, st = 0.f;
+      // in a half-height tile, columns 128-255 of each split are a second partial at row r + 128
+      const bool two = h0 >= 0 && r >= h0 && r < h0 + 128;
       for (int j = lane; j < n_vs; j += 32) {
         const float* b = part + (size_t)j * 5 * plane + r;
         merge_partial(ms, ss, as, mt, st, b[0], b[plane], b[2 * plane], b[3 * plane], b[4 * plane]);
+        if (two)
+          merge_partial(ms, ss, as, mt, st, b[128], b[plane + 128], b[2 * plane + 128], b[3 * plane + 128],
+                        b[4 * plane + 128]);
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {

@@ -25,7 +25,11 @@ struct Ctrl {
   uint32_t status;    // kDev* bits, cleared at the start of every call
   int32_t n_vsplit;   // vocabulary splits the forward used (written by the fused forward)
   int32_t work[4];    // work-unit counters: fused forward, fused backward, dH_s GEMM, dW_s GEMM; zeroed per call
-  int32_t pad[57];
+  // 1 + the first gathered row of a half-height last tile (0: none), written by the fused
+  // forward. In that tile the statistics of vocabulary columns 128-255 of row r sit in
+  // row r + 128 of the partials, which the readers of the partials merge into row r.
+  int32_t half_tile;
+  int32_t pad[56];
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

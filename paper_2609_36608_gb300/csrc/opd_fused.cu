@@ -31,6 +31,13 @@
 // CTAs' TMA completions are counted on the leader's barriers. Per byte staged
 // from L2 this does 1.5 times the MMA work of a single-CTA 128 x 256 tile (each
 // CTA stages half of W's rows).
+//
+// Half-height last tile: when the last row tile of a pair schedule holds at most
+// 128 supervised rows, its MMAs run with M = 128 (64 rows from each CTA), half the
+// tensor work. Each CTA's TMEM then holds its 64 rows twice: lanes 0-63 with
+// vocabulary columns 0-127 of the tile and lanes 64-127 with columns 128-255, in
+// TMEM columns 0-127. The forward stores the statistics of columns 128-255 of row r
+// as a second partial at row r + 128 (a padding row), which the readers merge.
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
@@ -69,11 +76,15 @@ struct FusedCfg {
 // vocabulary range start it together and stay together however their speeds differ.
 struct FusedSchedule {
   int n_rt, n_vt, n_vs, G, n_units;
+  int half_rt;  // row tile run at half height (M = 128 on a pair), or -1
 
   // Both passes walk the same units; only the forward keeps per-split statistics.
-  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split) {
+  // allow_half: on a CTA pair, a last row tile with at most half of its rows
+  // supervised runs as M = 128 MMAs (64 rows per CTA), half the tensor work.
+  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split, bool allow_half) {
     n_rt = (R + tile_rows - 1) / tile_rows;
     n_vt = (V + kBN - 1) / kBN;
+    half_rt = (allow_half && n_rt > 0 && R - (n_rt - 1) * tile_rows <= tile_rows / 2) ? n_rt - 1 : -1;
     // groups of at most G_ row tiles, as equal in size as possible
     G = G_ < 1 ? 1 : G_;
     if (n_rt > 0) {
@@ -408,8 +419,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int R = p.ctrl->R;
   FusedSchedule sch;
-  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit);
-  if (!BWD && blockIdx.x == 0 && threadIdx.x == 0) p.ctrl->n_vsplit = sch.n_vs;
+  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit, PAIR && p.half_tile != 0);
+  if (!BWD && blockIdx.x == 0 && threadIdx.x == 0) {
+    p.ctrl->n_vsplit = sch.n_vs;
+    p.ctrl->half_tile = sch.half_rt >= 0 ? sch.half_rt * C::kTileRows + 1 : 0;
+  }
   const int nks = (p.d_s + kKBlock - 1) / kKBlock;
   const int nkt = (p.d_t + kKBlock - 1) / kKBlock;
 
@@ -437,7 +451,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (u >= sch.n_units) break;
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
-        const int row0 = rt * C::kTileRows + (int)rank * kRowTile;
+        // a half-height tile takes 64 rows from each CTA (the MMA reads the first 64 staged)
+        const int row0 = rt * C::kTileRows + (int)rank * (rt == sch.half_rt ? kRowTile / 2 : kRowTile);
         for (int vt = vb; ok && vt < ve; ++vt) {
           const int wrow0 = vt * kBN + (int)rank * C::kBRows;
           for (int seg = 2 - HEADS; ok && seg < 2; ++seg) {  // teacher (two heads), then student
@@ -481,7 +496,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(C::kTileRows, kBN, false, false);
+      constexpr uint32_t idesc_full = idesc_bf16_f32(C::kTileRows, kBN, false, false);
+      constexpr uint32_t idesc_half = idesc_bf16_f32(C::kTileRows / 2, kBN, false, false);
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
@@ -494,6 +510,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (u >= sch.n_units) break;
         int rt, split, vb, ve;
         sch.unit(u, rt, split, vb, ve);
+        const uint32_t idesc = rt == sch.half_rt ? idesc_half : idesc_full;
         for (int vt = vb; ok && vt < ve; ++vt, ++lt) {
           for (int seg = 2 - HEADS; ok && seg < 2; ++seg) {
             // two heads: each segment reuses its columns every tile; one head: the
@@ -562,15 +579,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue
     const int ew = warp - 2;                 // epilogue warp index
     const int q = warp & 3;                  // TMEM lane quadrant this warp may access
-    const int half = ew / 4;                 // which 128 of the tile's 256 columns
-    const int cbase = half * kColsPerWarp;
-    const int row_in_tile = q * 32 + lane;
+    const int half = ew / 4;                 // which half of the accumulator's TMEM columns
     const uint32_t t_lane = (uint32_t)(q * 32) << 16;
     // the MMA issuer (in the pair's leader) waits for every epilogue warp of the pair
     const uint32_t t_free_addr = PAIR ? mapa_shared(smem_u32(t_free), 0u) : smem_u32(t_free);
     const uint32_t s_free_addr = PAIR ? mapa_shared(smem_u32(s_free), 0u) : smem_u32(s_free);
     int lt = 0, nu = 0;
     bool ok = true;
+    bool one_box = false;  // backward: the last tile stored only staging box 0
     const uint32_t stg = smem_u32(staging + ew * C::kStagingPerWarp);
     for (uint32_t k = 0; ok; ++k, ++nu) {
       const int u = take_unit_warp<PAIR>(k, unit_full, unit_empty, units, PAIR && rank != 0, status, lim);
@@ -581,8 +597,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (u >= sch.n_units) break;
       int rt, split, vb, ve;
       sch.unit(u, rt, split, vb, ve);
-      const int row_base = rt * C::kTileRows + (int)rank * kRowTile;
-      const int row = row_base + row_in_tile;
+      // Full tile: this CTA's 128 rows, lane quadrant q = rows 32q.., and this warp's
+      // 128 of the 256 columns. Half-height tile (M = 128 on the pair): this CTA's 64
+      // rows sit in lanes 0-63 with columns 0-127 and again in lanes 64-127 with columns
+      // 128-255, all in TMEM columns 0-127; this warp takes 64 of those columns.
+      const bool hm = rt == sch.half_rt;
+      const int drow0 = rt * C::kTileRows + (hm ? (int)rank * (kRowTile / 2) + (q & 1) * 32
+                                                : (int)rank * kRowTile + q * 32);
+      const int row = drow0 + lane;  // token row of this lane (rowc, dz)
       float ms = -INFINITY, Ss = 0.f, A = 0.f, mt = -INFINITY, St = 0.f;
       // backward row constants. Two heads: p_s = 2^(z_s k2 - b1), dz = p_s ((z_s - z_t) kc - cc).
       // One head: dz = coef (1[col = x] - p_s) with coef = rowc.y, token x = rowc.z (bits) and
@@ -611,19 +633,30 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
+        // TMEM column offset and tile column offset of this warp's columns
+        const int tcol = hm ? half * (kColsPerWarp / 2) : half * kColsPerWarp;
+        const int dcol = hm ? (q >> 1) * (kBN / 2) + tcol : tcol;
         if (HEADS == 1) {
           const int slot = lt & 1;
-          const int col0 = vt * kBN + cbase;
-          const uint32_t ts = (slot ? tmem_s : tmem_t) + t_lane + (uint32_t)cbase;
+          const int col0 = vt * kBN + dcol;
+          const uint32_t ts = (slot ? tmem_s : tmem_t) + t_lane + (uint32_t)tcol;
           if (!BWD) {
             const int nv = p.V - col0;
             fwd_chunk1<0>(ts, nv, p.k2, ms, Ss);
             fwd_chunk1<1>(ts, nv, p.k2, ms, Ss);
-            fwd_chunk1<2>(ts, nv, p.k2, ms, Ss);
-            fwd_chunk1<3>(ts, nv, p.k2, ms, Ss);
+            if (!hm) {
+              fwd_chunk1<2>(ts, nv, p.k2, ms, Ss);
+              fwd_chunk1<3>(ts, nv, p.k2, ms, Ss);
+            }
           } else {
-            const int x_rel = x_tok - col0;  // the token's column within this warp's 128
-            if (lane == 0) bulk_wait_read<1>();
+            const int x_rel = x_tok - col0;  // the token's column within this warp's columns
+            // staging box 0 is rewritten once its previous store has been read
+            if (lane == 0) {
+              if (one_box)
+                bulk_wait_read<0>();
+              else
+                bulk_wait_read<1>();
+            }
             __syncwarp();
             bwd_chunk1<0>(ts, p.k2, b1, kc, stg, lane);
             bwd_chunk1<1>(ts, p.k2, b1, kc, stg, lane);
@@ -631,20 +664,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, row_base + q * 32);
+              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, drow0);
               bulk_commit();
-              bulk_wait_read<1>();
+              if (!hm) bulk_wait_read<1>();
             }
             __syncwarp();
-            bwd_chunk1<2>(ts, p.k2, b1, kc, stg, lane);
-            bwd_chunk1<3>(ts, p.k2, b1, kc, stg, lane);
-            token_fixup(stg + 4096u, lane, x_rel - 64, at_token);
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, row_base + q * 32);
-              bulk_commit();
+            if (!hm) {
+              bwd_chunk1<2>(ts, p.k2, b1, kc, stg, lane);
+              bwd_chunk1<3>(ts, p.k2, b1, kc, stg, lane);
+              token_fixup(stg + 4096u, lane, x_rel - 64, at_token);
+              fence_proxy_async_smem();
+              __syncwarp();
+              if (lane == 0) {
+                tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, drow0);
+                bulk_commit();
+              }
             }
+            one_box = hm;
           }
           tc_fence_before();
           __syncwarp();
@@ -658,8 +694,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           continue;
         }
         // teacher columns to registers, then release them to the next tile's MMAs
-        uint32_t tv[kColsPerWarp];
-        tmem_ld128(tmem_t + t_lane + (uint32_t)cbase, tv);
+        uint32_t tv[kColsPerWarp];  // a half-height tile uses the first 64
+        tmem_ld128(tmem_t + t_lane + (uint32_t)tcol, tv);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
@@ -674,37 +710,48 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const int col0 = vt * kBN + cbase;
-        const uint32_t ts = tmem_s + t_lane + (uint32_t)cbase;
+        const int col0 = vt * kBN + dcol;
+        const uint32_t ts = tmem_s + t_lane + (uint32_t)tcol;
         if (!BWD) {
           const int nv = p.V - col0;
           fwd_chunk<0>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
           fwd_chunk<1>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
-          fwd_chunk<2>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
-          fwd_chunk<3>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+          if (!hm) {
+            fwd_chunk<2>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+            fwd_chunk<3>(ts, tv, nv, p.k2, ms, Ss, A, mt, St);
+          }
         } else {
           // staging box h of this warp is rewritten only after its previous TMA
-          // store has finished reading it
-          if (lane == 0) bulk_wait_read<1>();
+          // store has finished reading it (box 0 was the last store after a
+          // half-height tile, the second-to-last otherwise)
+          if (lane == 0) {
+            if (one_box)
+              bulk_wait_read<0>();
+            else
+              bulk_wait_read<1>();
+          }
           __syncwarp();
           bwd_chunk<0>(ts, tv, p.k2, b1, kc, cc, stg, lane);
           bwd_chunk<1>(ts, tv, p.k2, b1, kc, cc, stg, lane);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, row_base + q * 32);
+            tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, drow0);
             bulk_commit();
-            bulk_wait_read<1>();
+            if (!hm) bulk_wait_read<1>();
           }
           __syncwarp();
-          bwd_chunk<2>(ts, tv, p.k2, b1, kc, cc, stg, lane);
-          bwd_chunk<3>(ts, tv, p.k2, b1, kc, cc, stg, lane);
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, row_base + q * 32);
-            bulk_commit();
+          if (!hm) {
+            bwd_chunk<2>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+            bwd_chunk<3>(ts, tv, p.k2, b1, kc, cc, stg, lane);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, drow0);
+              bulk_commit();
+            }
           }
+          one_box = hm;
         }
         tc_fence_before();
         __syncwarp();
@@ -743,18 +790,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float mt1 = mb[3 * 32 + lane], St1 = mb[4 * 32 + lane];
         __syncwarp();
         if (lane == 0) mbar_arrive(&merge_empty[q]);
+        // In a half-height tile both warps of a quadrant may own no column of the unit's
+        // vocabulary range (its last tile, past V): the statistics then stay empty.
         const float Ms = fmaxf(ms, ms1);
-        const float f0 = ex2_ftz(ms - Ms), f1 = ex2_ftz(ms1 - Ms);
+        const bool any = Ms != -INFINITY;
+        const float f0 = any ? ex2_ftz(ms - Ms) : 0.f, f1 = any ? ex2_ftz(ms1 - Ms) : 0.f;
         Ss = Ss * f0 + Ss1 * f1;
         ms = Ms;
         const size_t plane = (size_t)p.T_pad;
-        float* base = p.partials + (size_t)split * 5 * plane + row;
+        // a half-height tile keeps the statistics of columns 128-255 at row + 128
+        const int srow = hm ? row + (q >> 1) * 128 : row;
+        float* base = p.partials + (size_t)split * 5 * plane + srow;
         base[0 * plane] = ms;
         base[1 * plane] = Ss;
         if (HEADS == 2) {
           const float Mt = fmaxf(mt, mt1);
           A = A * f0 + A1 * f1;
-          St = St * ex2_ftz(mt - Mt) + St1 * ex2_ftz(mt1 - Mt);
+          St = any ? St * ex2_ftz(mt - Mt) + St1 * ex2_ftz(mt1 - Mt) : 0.f;
           mt = Mt;
           base[2 * plane] = A;
           base[3 * plane] = mt;

@@ -39,6 +39,7 @@ struct FusedParams {
   int32_t max_vsplit;   // vocabulary splits the forward may use (<= kMaxVSplit; sizes partials)
   const float4* rowc;   // backward: [T_pad] = (lse_s log2 e, lse_s - lse_t + KL, g / tau, 0)
   int32_t mode;         // FusedMode; the W tensor maps' box height must be fused_w_box(mode)
+  int32_t half_tile;    // 1: on CTA pairs, a last row tile with at most 128 rows runs as M = 128 MMAs
 };
 
 inline int fused_mode(const FusedParams& p) { return p.mode == kFusedDefault ? kFusedDefaultMode : p.mode; }

@@ -49,6 +49,7 @@ __global__ void k_noalloc_rows(const uint8_t* __restrict__ mask, int32_t T) {
     ctrl->R = T;
     ctrl->status = 0u;
     ctrl->n_vsplit = 0;
+    ctrl->half_tile = 0;
   }
   if (threadIdx.x < 4) ctrl->work[threadIdx.x] = 0;
 }
@@ -151,6 +152,7 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.partials = partials;
   fp.max_vsplit = kSplits;
   fp.rowc = nullptr;
+  fp.half_tile = 1;
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
   if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
     return OPD_ERR_CUDA;

@@ -66,6 +66,7 @@ __global__ void k_head_rows(const HeadRowsParams p) {
   const int warps = (gridDim.x * blockDim.x) >> 5;
   const int R = p.ctrl->R;
   const int n_vs = p.ctrl->n_vsplit;
+  const int h0 = p.ctrl->half_tile - 1;  // first row of a half-height tile, or -1
   const size_t plane = (size_t)p.T_pad;
   for (int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < p.T; i += warps) {
     const int r = p.pos[i];
@@ -78,8 +79,13 @@ __global__ void k_head_rows(const HeadRowsParams p) {
       continue;
     }
     float m = -CUDART_INF_F, s = 0.f;
-    for (int j = lane; j < n_vs; j += 32) merge_stats(m, s, p.partials[(size_t)j * 5 * plane + r],
-                                                     p.partials[(size_t)j * 5 * plane + plane + r]);
+    // in a half-height tile, columns 128-255 of each split are a second partial at row r + 128
+    const bool two = h0 >= 0 && r >= h0 && r < h0 + 128;
+    for (int j = lane; j < n_vs; j += 32) {
+      const float* b = p.partials + (size_t)j * 5 * plane + r;
+      merge_stats(m, s, b[0], b[plane]);
+      if (two) merge_stats(m, s, b[128], b[plane + 128]);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float m2 = __shfl_xor_sync(0xffffffffu, m, o);

@@ -164,6 +164,24 @@ def test_random_shapes(lib, oracle_mod, case, monkeypatch):
     _full_check(lib, oracle_mod, w, mask=mask)
 
 
+@pytest.mark.parametrize("R", [1, 37, 128, 129, 293, 384])
+@pytest.mark.parametrize("half", ["1", "0"])
+def test_half_height_last_tile(lib, oracle_mod, monkeypatch, R, half):
+    """On CTA pairs a last row tile with at most 128 supervised rows runs as M = 128 MMAs
+    (64 rows per CTA; vocabulary columns 128-255 of each tile in TMEM lanes 64-127, their
+    statistics a second partial per row). R = 1, 37, 128 and 293 take that path, R = 129
+    and 384 do not; OPD_KL_HALF_TILE=0 runs every tile at full height. V = 4,986 leaves
+    122 columns in the last vocabulary tile, so with one tile per unit the warps of
+    columns 128-255 own no column there."""
+    monkeypatch.setenv("OPD_KL_FUSED", "pair256")
+    monkeypatch.setenv("OPD_KL_GEMM", "pair")
+    monkeypatch.setenv("OPD_KL_HALF_TILE", half)
+    w = _small_bf16(T=420, d_s=208, d_t=144, V=4986, tau=0.7, n_traj=1, traj_len=420, seed=31)
+    mask = np.zeros(w.T, np.uint8)
+    mask[np.random.default_rng(R).choice(w.T, R, replace=False)] = 1
+    _full_check(lib, oracle_mod, w, mask=mask)
+
+
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
     w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
                     seed=13)

@@ -168,15 +168,7 @@ def _random_cases(n, seed=4049):
                  tiling=["bn256/cta1", "pair256/pair"][i % 2], seed=200 + i) for i in range(n)]
 
 
-@pytest.mark.parametrize("case", _random_cases(8), ids=lambda c: f"T{c['T']}-d{c['d_s']}-V{c['V']}")
-def test_surrogate_and_scoring_random_shapes(lib, oracle_mod, case, monkeypatch):
-    fused, gemm = case["tiling"].split("/")
-    monkeypatch.setenv("OPD_KL_FUSED", fused)
-    monkeypatch.setenv("OPD_KL_GEMM", gemm)
-    w = _case(T=case["T"], d_s=case["d_s"], V=case["V"], tau=case["tau"], n_traj=1, traj_len=case["T"],
-              seed=case["seed"])
-    mask = (np.random.default_rng(case["seed"]).random(w.T) < case["density"]).astype(np.uint8)
-    mask[0] = 1
+def _score_and_surrogate_check(lib, oracle_mod, w, mask, seed):
     x = synth.hidden_and_heads(w, "cuda")
     tokens = synth.token_ids(w.seed, w.T, w.V)
     Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
@@ -186,9 +178,9 @@ def test_surrogate_and_scoring_random_shapes(lib, oracle_mod, case, monkeypatch)
     _close(lse[sup], ref_lse, 1e-4, 1e-4, "lse")
     _close(lp[sup], ref_lp, 1e-4, 1e-4, "logp")
     _, lp_full = oracle_mod.score(Hs, Ws, tokens, w.tau)
-    logp_old = (lp_full - _clear_offsets(case["seed"], w.T)).astype(np.float32)
-    adv = np.random.default_rng(case["seed"] + 1).choice([-1.0, 1.0], w.T) * \
-        np.random.default_rng(case["seed"] + 2).uniform(0.2, 1.5, w.T)
+    logp_old = (lp_full - _clear_offsets(seed, w.T)).astype(np.float32)
+    adv = np.random.default_rng(seed + 1).choice([-1.0, 1.0], w.T) * \
+        np.random.default_rng(seed + 2).uniform(0.2, 1.5, w.T)
     logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
     weights = np.where(sup, 1.0 / int(sup.sum()), 0.0).astype(np.float32)
     loss, _, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, mask, weights)
@@ -197,6 +189,31 @@ def test_surrogate_and_scoring_random_shapes(lib, oracle_mod, case, monkeypatch)
     _close(loss, ref.loss, 1e-4, 2e-3, "loss")
     assert _rel(dH, ref.dH_s) <= 1e-2, _rel(dH, ref.dH_s)
     assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
+
+
+@pytest.mark.parametrize("case", _random_cases(8), ids=lambda c: f"T{c['T']}-d{c['d_s']}-V{c['V']}")
+def test_surrogate_and_scoring_random_shapes(lib, oracle_mod, case, monkeypatch):
+    fused, gemm = case["tiling"].split("/")
+    monkeypatch.setenv("OPD_KL_FUSED", fused)
+    monkeypatch.setenv("OPD_KL_GEMM", gemm)
+    w = _case(T=case["T"], d_s=case["d_s"], V=case["V"], tau=case["tau"], n_traj=1, traj_len=case["T"],
+              seed=case["seed"])
+    mask = (np.random.default_rng(case["seed"]).random(w.T) < case["density"]).astype(np.uint8)
+    mask[0] = 1
+    _score_and_surrogate_check(lib, oracle_mod, w, mask, case["seed"])
+
+
+@pytest.mark.parametrize("R", [1, 100, 128, 129, 300])
+def test_surrogate_and_scoring_half_height_last_tile(lib, oracle_mod, monkeypatch, R):
+    """The single-head kernels on CTA pairs with a last row tile of at most 128 supervised
+    rows (R = 1, 100, 128, 300) run it as M = 128 MMAs; R = 129 does not. V = 2,100 leaves 52
+    columns in the last vocabulary tile."""
+    monkeypatch.setenv("OPD_KL_FUSED", "pair256")
+    monkeypatch.setenv("OPD_KL_GEMM", "pair")
+    w = _case(T=360, d_s=136, V=2100, tau=0.8, n_traj=1, traj_len=360, seed=41)
+    mask = np.zeros(w.T, np.uint8)
+    mask[np.random.default_rng(R).choice(w.T, R, replace=False)] = 1
+    _score_and_surrogate_check(lib, oracle_mod, w, mask, 41 + R)
 
 
 def test_surrogate_on_policy_and_accumulate(lib, oracle_mod):
