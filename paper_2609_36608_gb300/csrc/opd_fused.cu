@@ -97,15 +97,17 @@ struct FusedSchedule {
       // fewest tiles on the busiest worker, then the fewest splits; at least enough
       // splits that the units running at once span one raster group of row tiles, so
       // the group's hidden-state tiles stay in L2 (with fewer splits every worker
-      // streams the whole vocabulary against its own row tile and H leaves L2)
+      // streams the whole vocabulary against its own row tile and H leaves L2).
+      // Work is counted in half units: a half-height tile's units cost half.
       long best = -1;
       const int cap = max_split < 1 ? 1 : (max_split > kMaxVSplit ? kMaxVSplit : max_split);
       const int max_vs = n_vt < cap ? n_vt : cap;
       int min_vs = (workers + G - 1) / G;
       min_vs = min_vs < 1 ? 1 : (min_vs > max_vs ? max_vs : min_vs);
       n_vs = min_vs;
+      const long rows2 = 2L * n_rt - (half_rt >= 0 ? 1 : 0);
       for (int s = min_vs; s <= max_vs; ++s) {
-        const long waves = ((long)n_rt * s + workers - 1) / workers;
+        const long waves = (rows2 * s + 2L * workers - 1) / (2L * workers);
         const long cost = waves * ((n_vt + s - 1) / s);
         if (best < 0 || cost < best) {
           best = cost;
