@@ -5,8 +5,8 @@ all, such as a host process that owns the whole GPU through its own fixed pool
 and forbids libraries from calling cudaMalloc. It keeps its scratch in a fixed
 array inside the library instead of a caller-provided workspace. This file
 checks it through the C ABI against opd_kl_forward, with the same tolerance as
-the parity tests, on two calls in a row with different problems (the second
-call reuses the array the first one left behind). It runs last so that a
+the parity tests, on three calls in a row with different problems (each call
+reuses the array the previous one left behind). It runs last so that a
 failure here leaves every other test already run.
 """
 
@@ -53,10 +53,13 @@ def _both(lib, w):
     return lay.mask != 0, kl.cpu().numpy(), st.cpu().numpy(), kl_ref.cpu().numpy(), st_ref.cpu().numpy()
 
 
-def test_noalloc_forward_matches_workspace_forward_on_two_calls(lib):
+def test_noalloc_forward_matches_workspace_forward_on_three_calls(lib):
+    # every row is scheduled here (no compaction): T = 300 leaves a last row tile of 44 rows,
+    # which runs at half height on a CTA pair
     cases = [_case("noalloc_a", T=700, seed=21),
              _case("noalloc_b", T=lib.OPD_KL_NOALLOC_MAX_ROWS, d_s=128, d_t=192, V=1237, tau=1.0, seed=22,
-                   traj_len=512)]
+                   traj_len=512),
+             _case("noalloc_c", T=300, d_s=192, d_t=256, V=3000, tau=1.3, seed=23, traj_len=300)]
     for w in cases:
         sup, kl, st, kl_ref, st_ref = _both(lib, w)
         excess = np.abs(kl - kl_ref) - (KL_ABS + KL_REL * np.abs(kl_ref))
