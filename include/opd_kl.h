@@ -50,8 +50,10 @@
  *                               256 x 256 tiles on a CTA pair (default)
  *   OPD_KL_GEMM=cta1|pair       gradient-GEMM tiling, same two choices (default pair)
  *   OPD_KL_GROUP_ROWS=n         row tiles walked together in L2 (default 10)
- *   OPD_KL_HALF_TILE=0|1        on CTA pairs, a last row tile with at most 128 supervised
- *                               rows runs at half height, M = 128 (default 1)
+ *   OPD_KL_HALF_TILE=0|1        on CTA pairs, a last row tile with at most 128 rows runs at
+ *                               half height, M = 128, in the fused kernels and GEMMs (default 1)
+ *   OPD_KL_VSPLIT=n             exactly n vocabulary splits in the fused kernels (default 0:
+ *                               searched)
  *   OPD_KL_MAX_KSPLIT=n         largest K split of the dH_s GEMM (default 16)
  *   OPD_KL_DETERMINISTIC=1      bit-reproducible dH_s: no split-K reduce-adds (KL, stats and
  *                               dW_s are bit-reproducible in every mode); the dH_s GEMM then

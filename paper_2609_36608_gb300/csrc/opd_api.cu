@@ -331,6 +331,7 @@ FusedParams fused_params(const Call& c) {
   fp.mode = fused_tile_mode();
   fp.max_vsplit = kMaxVSplit;
   fp.half_tile = env_int("OPD_KL_HALF_TILE", 1) != 0 ? 1 : 0;
+  fp.vsplit = env_int("OPD_KL_VSPLIT", 0);
   return fp;
 }
 
@@ -414,6 +415,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumul
   gh.reduce = deterministic ? 0 : 1;
   gh.pair = gemm_pair_mode();
   gh.work_slot = 2;
+  gh.half_tile = env_int("OPD_KL_HALF_TILE", 1) != 0 ? 1 : 0;
   gh.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dH", c.s, [&] { return launch_gemm(false, true, m.dz_a_k, m.ws_b_mn, m.dhg, gh, c.dev.sm_count, c.s); }));
 
@@ -428,6 +430,7 @@ opd_status gradient_gemms(const Call& c, const Maps& m, float* dH_s, int accumul
   gw.reduce = accumulate_dW ? 1 : 0;
   gw.pair = gemm_pair_mode();
   gw.work_slot = 3;
+  gw.half_tile = gh.half_tile;
   gw.wait_limit_ns = kDefaultWaitLimitNs;
   OPD_CUDA(timed("gemm_dW", c.s, [&] { return launch_gemm(true, true, m.dz_a_mn, m.hsg_b_mn, m.dw, gw, c.dev.sm_count, c.s); }));
 

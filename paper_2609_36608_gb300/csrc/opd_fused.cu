@@ -81,7 +81,8 @@ struct FusedSchedule {
   // Both passes walk the same units; only the forward keeps per-split statistics.
   // allow_half: on a CTA pair, a last row tile with at most half of its rows
   // supervised runs as M = 128 MMAs (64 rows per CTA), half the tensor work.
-  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split, bool allow_half) {
+  __device__ void init(int R, int V, int tile_rows, int workers, int G_, int max_split, bool allow_half,
+                       int force_split) {
     n_rt = (R + tile_rows - 1) / tile_rows;
     n_vt = (V + kBN - 1) / kBN;
     half_rt = (allow_half && n_rt > 0 && R - (n_rt - 1) * tile_rows <= tile_rows / 2) ? n_rt - 1 : -1;
@@ -91,23 +92,27 @@ struct FusedSchedule {
       const int n_groups = (n_rt + G - 1) / G;
       G = (n_rt + n_groups - 1) / n_groups;
     }
+    const int cap = max_split < 1 ? 1 : (max_split > kMaxVSplit ? kMaxVSplit : max_split);
+    const int max_vs = n_vt < cap ? n_vt : cap;
     if (n_rt == 0) {
       n_vs = 1;
+    } else if (force_split > 0) {
+      n_vs = force_split < max_vs ? force_split : max_vs;
     } else {
       // fewest tiles on the busiest worker, then the fewest splits; at least enough
       // splits that the units running at once span one raster group of row tiles, so
       // the group's hidden-state tiles stay in L2 (with fewer splits every worker
       // streams the whole vocabulary against its own row tile and H leaves L2).
-      // Work is counted in half units: a half-height tile's units cost half.
+      // A half-height tile still counts as a full one here: counted as half, the search
+      // at the 1.7B size picks 75 splits instead of 33, whose unequal unit lengths break
+      // the lockstep of the pairs sharing a range and cost more DRAM reads than the
+      // balance gains (measured).
       long best = -1;
-      const int cap = max_split < 1 ? 1 : (max_split > kMaxVSplit ? kMaxVSplit : max_split);
-      const int max_vs = n_vt < cap ? n_vt : cap;
       int min_vs = (workers + G - 1) / G;
       min_vs = min_vs < 1 ? 1 : (min_vs > max_vs ? max_vs : min_vs);
       n_vs = min_vs;
-      const long rows2 = 2L * n_rt - (half_rt >= 0 ? 1 : 0);
       for (int s = min_vs; s <= max_vs; ++s) {
-        const long waves = (rows2 * s + 2L * workers - 1) / (2L * workers);
+        const long waves = ((long)n_rt * s + workers - 1) / workers;
         const long cost = waves * ((n_vt + s - 1) / s);
         if (best < 0 || cost < best) {
           best = cost;
@@ -421,7 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int R = p.ctrl->R;
   FusedSchedule sch;
-  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit, PAIR && p.half_tile != 0);
+  sch.init(R, p.V, C::kTileRows, n_workers, p.group_rows, p.max_vsplit, PAIR && p.half_tile != 0, p.vsplit);
   if (!BWD && blockIdx.x == 0 && threadIdx.x == 0) {
     p.ctrl->n_vsplit = sch.n_vs;
     p.ctrl->half_tile = sch.half_rt >= 0 ? sch.half_rt * C::kTileRows + 1 : 0;

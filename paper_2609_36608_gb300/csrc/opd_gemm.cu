@@ -45,11 +45,17 @@ struct GemmCfg {
 
 struct GemmSchedule {
   int n_mt, n_nt, nkb, n_ks, n_units;
+  int half_mt;  // M tile run at half height (M = 128 on a pair), or -1
 
-  __device__ void init(int M, int N, int K, int tile_rows, int grid, int max_ks) {
+  // allow_half: on a CTA pair, a last M tile with at most half of its rows in range runs
+  // as M = 128 MMAs (64 rows per CTA). The split search still counts it as a full tile:
+  // counting it as half picks more K splits (16 instead of 9 for dH_s at the 1.7B size),
+  // whose extra reduce-adds cost more than the better balance gains (measured).
+  __device__ void init(int M, int N, int K, int tile_rows, int grid, int max_ks, bool allow_half) {
     n_mt = (M + tile_rows - 1) / tile_rows;
     n_nt = (N + kBN - 1) / kBN;
     nkb = (K + kKBlock - 1) / kKBlock;
+    half_mt = (allow_half && n_mt > 0 && M - (n_mt - 1) * tile_rows <= tile_rows / 2) ? n_mt - 1 : -1;
     n_ks = 1;
     if (max_ks > 1 && n_mt > 0 && nkb > 1) {
       long best = -1;
@@ -155,7 +161,7 @@ __global__ void __launch_bounds__(192, 1)
   const int M = p.m_is_R ? R : p.M;
   const int K = p.k_is_R ? R : p.K;
   GemmSchedule sch;
-  sch.init(M, p.N, K, C::kTileRows, n_workers, p.max_ksplit);
+  sch.init(M, p.N, K, C::kTileRows, n_workers, p.max_ksplit, PAIR && p.half_tile != 0);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -184,8 +190,8 @@ __global__ void __launch_bounds__(192, 1)
         if (u >= sch.n_units) break;
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
-        // this CTA's 128 rows of A and (pair) its half of B's columns
-        const int m0 = mt * C::kTileRows + (int)rank * kRowTile;
+        // this CTA's 128 rows of A (64 used in a half-height tile) and (pair) its half of B's columns
+        const int m0 = mt * C::kTileRows + (int)rank * (mt == sch.half_mt ? kRowTile / 2 : kRowTile);
         const int n0 = nt * kBN + (int)rank * (kBN - C::kBCols);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, status, lim)) {
@@ -237,7 +243,8 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(C::kTileRows, kBN, A_MN, B_MN);
+      constexpr uint32_t idesc_full = idesc_bf16_f32(C::kTileRows, kBN, A_MN, B_MN);
+      constexpr uint32_t idesc_half = idesc_bf16_f32(C::kTileRows / 2, kBN, A_MN, B_MN);
       uint32_t stage = 0, phase = 0;
       int lt = 0;
       bool ok = true;
@@ -251,6 +258,7 @@ __global__ void __launch_bounds__(192, 1)
         if (u >= sch.n_units) break;
         int mt, nt, kb0, kb1;
         sch.unit(u, mt, nt, kb0, kb1);
+        const uint32_t idesc = mt == sch.half_mt ? idesc_half : idesc_full;
         const int buf = lt & 1;
         const uint32_t acc_par = (uint32_t)(lt >> 1) & 1u;
         if (!mbar_wait(&acc_empty[buf], acc_par ^ 1u, status, lim)) {
@@ -321,11 +329,17 @@ __global__ void __launch_bounds__(192, 1)
       if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[buf], acc_par, status, lim))) break;
       tc_fence_after();
       const bool empty_k = kb1 <= kb0;
-      const int m0 = mt * C::kTileRows + (int)rank * kRowTile + q * 32, n0 = nt * kBN;
+      // Full tile: this CTA's rows 32q.. over all 256 columns. Half-height tile: the CTA's
+      // 64 rows sit in lanes 0-63 with columns 0-127 and in lanes 64-127 with columns
+      // 128-255, all in TMEM columns 0-127.
+      const bool hm = mt == sch.half_mt;
+      const int m0 = mt * C::kTileRows + (hm ? (int)rank * (kRowTile / 2) + (q & 1) * 32 : (int)rank * kRowTile + q * 32);
+      const int n0 = nt * kBN + (hm ? (q >> 1) * (kBN / 2) : 0);
+      const int n_chunks = hm ? kBN / 64 : kBN / 32;
       // rows of the last tile past M (a pair's odd CTA can hold none) are not stored
       if (!(empty_k && p.reduce) && m0 < M) {
 #pragma unroll 1
-        for (int c = 0; c < kBN / 32; ++c) {
+        for (int c = 0; c < n_chunks; ++c) {
           if (n0 + c * 32 >= p.N) break;
           uint32_t r[32];
           if (!empty_k) {

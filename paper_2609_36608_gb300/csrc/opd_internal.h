@@ -40,6 +40,7 @@ struct FusedParams {
   const float4* rowc;   // backward: [T_pad] = (lse_s log2 e, lse_s - lse_t + KL, g / tau, 0)
   int32_t mode;         // FusedMode; the W tensor maps' box height must be fused_w_box(mode)
   int32_t half_tile;    // 1: on CTA pairs, a last row tile with at most 128 rows runs as M = 128 MMAs
+  int32_t vsplit;       // > 0: exactly this many vocabulary splits (capped by max_vsplit); 0: searched
 };
 
 inline int fused_mode(const FusedParams& p) { return p.mode == kFusedDefault ? kFusedDefaultMode : p.mode; }
@@ -52,6 +53,7 @@ struct GemmParams {
   int32_t reduce;       // 1 = TMA reduce-add into C, 0 = TMA store
   int32_t pair;         // 1 = 256 x 256 tiles on CTA pairs (B must be MN-major), 0 = 128 x 256 on one CTA
   int32_t work_slot;    // pairs: the Ctrl::work counter this launch takes its tiles from (2 or 3)
+  int32_t half_tile;    // 1: on CTA pairs, a last M tile with at most 128 rows runs as M = 128 MMAs
   uint64_t wait_limit_ns;
 };
 

@@ -153,6 +153,7 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.max_vsplit = kSplits;
   fp.rowc = nullptr;
   fp.half_tile = 1;
+  fp.vsplit = 0;
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
   if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
     return OPD_ERR_CUDA;
