@@ -182,6 +182,24 @@ def test_half_height_last_tile(lib, oracle_mod, monkeypatch, R, half):
     _full_check(lib, oracle_mod, w, mask=mask)
 
 
+@pytest.mark.parametrize("env", [("OPD_KL_VSPLIT", "1"), ("OPD_KL_VSPLIT", "7"), ("OPD_KL_VSPLIT", "128"),
+                                 ("OPD_KL_GROUP_ROWS", "1"), ("OPD_KL_GROUP_ROWS", "64"),
+                                 ("OPD_KL_MAX_KSPLIT", "1"), ("OPD_KL_MAX_KSPLIT", "16")],
+                         ids=lambda e: f"{e[0]}={e[1]}")
+def test_tuning_overrides_keep_parity(lib, oracle_mod, monkeypatch, env):
+    """Every schedule the tuning overrides reach computes the same result: one vocabulary split
+    (a unit walks all of V), the largest split count, raster groups of one row tile or of all
+    of them, and the dH_s GEMM with and without split-K. Four row-pair tiles, the last one at
+    half height (R = 800)."""
+    monkeypatch.setenv("OPD_KL_FUSED", "pair256")
+    monkeypatch.setenv("OPD_KL_GEMM", "pair")
+    monkeypatch.setenv(*env)
+    w = _small_bf16(T=1000, d_s=128, d_t=192, V=3000, tau=1.0, n_traj=1, traj_len=1000, seed=37)
+    mask = np.zeros(w.T, np.uint8)
+    mask[np.random.default_rng(37).choice(w.T, 800, replace=False)] = 1
+    _full_check(lib, oracle_mod, w, mask=mask)
+
+
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
     w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
                     seed=13)
