@@ -15,53 +15,79 @@ namespace opd {
 namespace {
 
 constexpr int kCompactThreads = 1024;
+constexpr int kCompactPer = 16;  // mask bytes per thread and pass (one 16-byte load when aligned)
 
-// One CTA: each thread counts the mask over a contiguous slice, a block-wide
-// exclusive scan gives each slice its output offset, then the slice is written.
+// One CTA walks the mask in passes of kCompactThreads x 16 rows: each thread takes 16
+// consecutive rows, a block-wide exclusive scan of the per-thread counts gives each
+// thread its output offset, and a running total carries the offset to the next pass.
+// Loads are coalesced (16-byte vectors when the mask is 16-byte aligned, bytes
+// otherwise) and pos is written four rows per 16-byte store.
 __global__ void __launch_bounds__(kCompactThreads)
     k_compact(const uint8_t* __restrict__ mask, int32_t T, int32_t* __restrict__ idx, int32_t* __restrict__ pos,
               Ctrl* ctrl) {
   __shared__ int32_t warp_tot[32];
   const int tid = threadIdx.x;
+  const int lane = tid & 31, w = tid >> 5;
   if (tid == 0) ctrl->status = 0u;
   if (tid < 4) ctrl->work[tid] = 0;
-  const int per = (T + kCompactThreads - 1) / kCompactThreads;
-  const int lo = min(T, tid * per);
-  const int hi = min(T, lo + per);
-  int cnt = 0;
-  for (int i = lo; i < hi; ++i) cnt += mask[i] != 0;
-  // inclusive warp scan, then scan of warp totals
-  const int lane = tid & 31, w = tid >> 5;
-  int x = cnt;
+  const bool vec = (reinterpret_cast<uintptr_t>(mask) & 15u) == 0;
+  int carry = 0;  // supervised rows before this pass
+  for (int base = 0; base < T; base += kCompactThreads * kCompactPer) {
+    const int lo = base + tid * kCompactPer;
+    uint32_t bits = 0;  // bit j: row lo + j is supervised
+    if (vec && lo + kCompactPer <= T) {
+      const uint4 v = *reinterpret_cast<const uint4*>(mask + lo);
+      const uint32_t wv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) warp_tot[w] = x;
-  __syncthreads();
-  if (w == 0) {
-    int t = warp_tot[lane];
+      for (int j = 0; j < kCompactPer; ++j) bits |= (((wv[j >> 2] >> (8 * (j & 3))) & 0xFFu) != 0u ? 1u : 0u) << j;
+    } else {
+#pragma unroll
+      for (int j = 0; j < kCompactPer; ++j)
+        if (lo + j < T && mask[lo + j] != 0) bits |= 1u << j;
+    }
+    const int cnt = __popc(bits);
+    // inclusive warp scan, then scan of the warp totals
+    int x = cnt;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, t, o);
-      if (lane >= o) t += y;
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
     }
-    warp_tot[lane] = t;  // inclusive totals
-  }
-  __syncthreads();
-  int off = x - cnt + (w > 0 ? warp_tot[w - 1] : 0);
-  for (int i = lo; i < hi; ++i) {
-    if (mask[i] != 0) {
-      idx[off] = i;
-      pos[i] = off;
-      ++off;
+    __syncthreads();  // warp_tot of the previous pass has been read
+    if (lane == 31) warp_tot[w] = x;
+    __syncthreads();
+    if (w == 0) {
+      int t = warp_tot[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, t, o);
+        if (lane >= o) t += y;
+      }
+      warp_tot[lane] = t;  // inclusive totals
+    }
+    __syncthreads();
+    int off = carry + x - cnt + (w > 0 ? warp_tot[w - 1] : 0);
+    int pv[kCompactPer];
+#pragma unroll
+    for (int j = 0; j < kCompactPer; ++j) {
+      if ((bits >> j) & 1u) {
+        idx[off] = lo + j;
+        pv[j] = off++;
+      } else {
+        pv[j] = -1;
+      }
+    }
+    if (lo + kCompactPer <= T) {  // pos is 16-byte aligned (workspace) and lo a multiple of 16
+#pragma unroll
+      for (int j = 0; j < kCompactPer; j += 4)
+        *reinterpret_cast<int4*>(pos + lo + j) = make_int4(pv[j], pv[j + 1], pv[j + 2], pv[j + 3]);
     } else {
-      pos[i] = -1;
+      for (int j = 0; j < kCompactPer && lo + j < T; ++j) pos[lo + j] = pv[j];
     }
+    carry += warp_tot[31];
   }
-  if (tid == kCompactThreads - 1) {
-    ctrl->R = warp_tot[31];
+  if (tid == 0) {
+    ctrl->R = carry;
     ctrl->n_vsplit = 0;
     ctrl->half_tile = 0;
   }
