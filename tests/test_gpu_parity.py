@@ -200,6 +200,33 @@ def test_tuning_overrides_keep_parity(lib, oracle_mod, monkeypatch, env):
     _full_check(lib, oracle_mod, w, mask=mask)
 
 
+def test_mask_at_any_byte_offset(lib):
+    """The compaction reads the mask in 16-byte vectors when it is 16-byte aligned and byte by
+    byte otherwise (a mask that is a slice of a larger one, as with row chunks): both give
+    bit-identical results."""
+    w = _small_bf16(T=1000, d_s=64, d_t=64, V=700, tau=1.0, n_traj=10, traj_len=100, seed=38)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    outs = []
+    for offset in (0, 5):
+        backing = torch.zeros(w.T + 16, dtype=torch.uint8, device="cuda")
+        backing[offset:offset + w.T] = torch.from_numpy(lay.mask).cuda()
+        mask = backing[offset:offset + w.T]
+        assert (mask.data_ptr() % 16 == 0) == (offset == 0)
+        kl = torch.full((w.T,), float("nan"), device="cuda")
+        st = torch.full((w.T, 3), float("nan"), device="cuda")
+        lib.opd_kl_forward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, kl, st, ws)
+        torch.cuda.synchronize()
+        assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+        outs.append((kl.cpu().numpy(), st.cpu().numpy()))
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
+    np.testing.assert_array_equal(outs[0][1], outs[1][1])
+    sup = lay.mask != 0
+    assert (outs[0][0][~sup] == 0).all() and (outs[0][0][sup] > 0).all()
+
+
 def test_bf16_correlated_teacher_small_kl(lib, oracle_mod):
     w = _small_bf16(T=256, d_s=128, d_t=320, V=2048, tau=1.0, n_traj=2, traj_len=128, correlated_teacher=True,
                     seed=13)
