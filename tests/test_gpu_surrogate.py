@@ -287,3 +287,56 @@ def test_full_size_surrogate_and_scoring_sampled_rows(lib, oracle_mod, name):
     ref2 = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
                                 mask2, weights.astype(np.float64), w.tau, rows=pick[::2], want_dH=False)
     assert _rel(dW2, ref2.dW_s) <= 1e-2, _rel(dW2, ref2.dW_s)
+
+
+def test_surrogate_loss_step_in_a_cuda_graph(lib):
+    """The whole surrogate loss step (weights on the device, surrogate forward and backward,
+    batch loss) makes no host synchronisation, so it captures into one CUDA graph; a replay
+    reproduces the eager step."""
+    w = _case(T=600, d_s=128, V=3000, tau=1.0, n_traj=6, traj_len=100, seed=43)
+    lay = synth.layout(w)
+    n_ids = int(lay.seg_id.max()) + 1
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = torch.from_numpy(synth.token_ids(w.seed, w.T, w.V)).cuda()
+    rng = np.random.default_rng(43)
+    logp_teacher = torch.from_numpy((rng.standard_normal(w.T) - 7.0).astype(np.float32)).cuda()
+    logp_old = logp_teacher + torch.from_numpy((0.3 * rng.standard_normal(w.T)).astype(np.float32)).cuda()
+    mask = torch.from_numpy(lay.mask).cuda()
+    seg = torch.from_numpy(lay.seg_id).cuda()
+    prob = lib.make_problem(w.T, w.d_s, w.d_s, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws = lib.allocate_workspace(prob)
+    seq_ws = torch.empty(lib.opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8, device="cuda")
+    wts = torch.empty(w.T, device="cuda")
+    loss = torch.empty(w.T, device="cuda")
+    lp = torch.empty(w.T, device="cuda")
+    dH = torch.empty(w.T, w.d_s, device="cuda")
+    dW = torch.empty(w.V, w.d_s, device="cuda")
+    total = torch.empty(1, device="cuda")
+
+    def step():
+        lib.opd_seq_mean_token_mean_device(seg, mask, n_ids, 1e-8, None, wts, None, seq_ws)
+        lib.opd_surrogate_fwd_bwd(prob, x["H_s"], x["W_s"], tokens, logp_old, logp_teacher, mask, wts, loss, lp,
+                                  dH, dW, False, ws)
+        lib.opd_seq_mean_token_mean_device(seg, mask, n_ids, 1e-8, loss, None, total, seq_ws)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()  # eager step, outside the capture (kernel attributes are set here)
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK and lib.opd_kl_get_status(seq_ws) == lib.OPD_OK
+    eager = {k: v.clone() for k, v in dict(loss=loss, lp=lp, dH=dH, dW=dW, total=total).items()}
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for t in (loss, lp, dH, dW, total):
+        t.fill_(float("nan"))
+    graph.replay()
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK and lib.opd_kl_get_status(seq_ws) == lib.OPD_OK
+    for k in ("loss", "lp", "dW"):
+        np.testing.assert_array_equal(dict(loss=loss, lp=lp, dW=dW)[k].cpu().numpy(), eager[k].cpu().numpy())
+    # dH_s: split-K partial sums in arrival order; L: a double sum over blocks in arrival order
+    assert _rel(dH.cpu().numpy(), eager["dH"].cpu().numpy().astype(np.float64)) < 1e-5
+    assert np.isfinite(total.item()) and abs(total.item() - eager["total"].item()) <= 1e-6 * abs(eager["total"].item())
