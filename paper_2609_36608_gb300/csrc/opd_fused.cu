@@ -49,6 +49,11 @@ constexpr int kBN = 256;   // vocabulary columns per tile (MMA N)
 constexpr int kNEpi = 8;   // epilogue warps
 constexpr int kColsPerWarp = kBN / 2;
 constexpr int kThreads = 64 + 32 * kNEpi;
+// Backward: 64-column bf16 dz staging boxes per epilogue warp (4 KB each). With one box
+// the warp waits for each TMA store to read it before refilling it, and the 32 KB saved
+// buy a sixth pipeline stage: the backward ran 2.2% faster than with two boxes and five
+// stages (the single-head backward 4.9%).
+constexpr int kDzBoxes = 1;
 
 template <bool BWD, bool PAIR, int HEADS>
 struct FusedCfg {
@@ -57,7 +62,7 @@ struct FusedCfg {
   static constexpr uint32_t kABytes = kRowTile * kKBlock * 2;
   static constexpr uint32_t kBBytes = kBRows * kKBlock * 2;
   static constexpr uint32_t kStageBytes = kABytes + kBBytes;
-  static constexpr uint32_t kStagingPerWarp = BWD ? 32 * kColsPerWarp * 2 : 0;  // bf16 dz rows of one warp
+  static constexpr uint32_t kStagingPerWarp = BWD ? 32 * 64 * 2 * kDzBoxes : 0;  // bf16 dz boxes of one warp
   static constexpr uint32_t kMergeBytes = BWD ? 0 : 4 * 5 * 32 * 4;             // per quadrant 5 x 32
   static constexpr uint32_t kBarrierBytes = 512;
   static constexpr size_t kFixed = 1024 + (size_t)kNEpi * kStagingPerWarp + kMergeBytes + kBarrierBytes;
@@ -253,7 +258,7 @@ __device__ __forceinline__ void bwd_chunk(uint32_t ts, const uint32_t (&tv)[kCol
     }
     w[j] = pack_bf16x2(dz2[0], dz2[1]);
   }
-  const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
+  const uint32_t box = stg + (uint32_t)((C >> 1) % kDzBoxes) * 4096u;
   const uint32_t jb = (uint32_t)(C & 1) * 4u;
 #pragma unroll
   for (int jj = 0; jj < 4; ++jj)
@@ -321,7 +326,7 @@ __device__ __forceinline__ void bwd_chunk1(uint32_t ts, float k2, float b1, floa
     f2_unpack(f2_mul(ncoef2, f2_pack(ex2_ftz(a), ex2_ftz(b))), a, b);
     w[j] = pack_bf16x2(a, b);
   }
-  const uint32_t box = stg + (uint32_t)(C >> 1) * 4096u;
+  const uint32_t box = stg + (uint32_t)((C >> 1) % kDzBoxes) * 4096u;
   const uint32_t jb = (uint32_t)(C & 1) * 4u;
 #pragma unroll
   for (int jj = 0; jj < 4; ++jj)
@@ -659,7 +664,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int x_rel = x_tok - col0;  // the token's column within this warp's columns
             // staging box 0 is rewritten once its previous store has been read
             if (lane == 0) {
-              if (one_box)
+              if (one_box || kDzBoxes == 1)
                 bulk_wait_read<0>();
               else
                 bulk_wait_read<1>();
@@ -673,17 +678,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) {
               tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, drow0);
               bulk_commit();
-              if (!hm) bulk_wait_read<1>();
+              if (!hm) bulk_wait_read<kDzBoxes - 1>();
             }
             __syncwarp();
             if (!hm) {
+              constexpr uint32_t box1 = kDzBoxes > 1 ? 4096u : 0u;
               bwd_chunk1<2>(ts, p.k2, b1, kc, stg, lane);
               bwd_chunk1<3>(ts, p.k2, b1, kc, stg, lane);
-              token_fixup(stg + 4096u, lane, x_rel - 64, at_token);
+              token_fixup(stg + box1, lane, x_rel - 64, at_token);
               fence_proxy_async_smem();
               __syncwarp();
               if (lane == 0) {
-                tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, drow0);
+                tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + box1, col0 + 64, drow0);
                 bulk_commit();
               }
             }
@@ -732,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // store has finished reading it (box 0 was the last store after a
           // half-height tile, the second-to-last otherwise)
           if (lane == 0) {
-            if (one_box)
+            if (one_box || kDzBoxes == 1)
               bulk_wait_read<0>();
             else
               bulk_wait_read<1>();
@@ -745,16 +751,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (lane == 0) {
             tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp, col0, drow0);
             bulk_commit();
-            if (!hm) bulk_wait_read<1>();
+            if (!hm) bulk_wait_read<kDzBoxes - 1>();
           }
           __syncwarp();
           if (!hm) {
+            constexpr uint32_t box1 = kDzBoxes > 1 ? 4096u : 0u;
             bwd_chunk<2>(ts, tv, p.k2, b1, kc, cc, stg, lane);
             bwd_chunk<3>(ts, tv, p.k2, b1, kc, cc, stg, lane);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + 4096, col0 + 64, drow0);
+              tma_store_2d(&tm_dz, staging + ew * C::kStagingPerWarp + box1, col0 + 64, drow0);
               bulk_commit();
             }
           }
