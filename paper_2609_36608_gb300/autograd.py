@@ -9,6 +9,12 @@ OPDSeqMeanKLLoss: the paper's batch loss over the per-token KL (Appendix B.4,
 seq-mean-token-mean), computed with its gradients by one opd_kl_seq_mean_fwd_bwd call in
 the forward; the backward scales those gradients by the upstream scalar.
 
+OPDSurrogateLoss: the sampled-token dual-clip surrogate the paper optimises (Appendix B.4,
+Eq. opd-token-advantage, opd-ratio, opd-dual-clip, opd-surrogate) with seq-mean-token-mean
+weights computed on the device; one opd_surrogate_fwd_bwd call in the forward, the
+backward scales its gradients. score_tokens: the frozen teacher's log-partition and token
+log-probabilities (no gradient).
+
 Gradients come back in the dtype of the tensors they belong to (autograd's rule); the
 library computes them in float32.
 """
@@ -97,3 +103,63 @@ class OPDSeqMeanKLLoss(torch.autograd.Function):
         dH, dW = ctx.saved_tensors
         g = grad_loss.float()
         return (dH * g).to(ctx.dtypes[0]), None, (dW * g).to(ctx.dtypes[1]), None, None, None, None, None, None
+
+
+class OPDSurrogateLoss(torch.autograd.Function):
+    """loss = OPDSurrogateLoss.apply(H_s, W_s, tokens, logp_old, logp_teacher, mask, seg_id, n_ids,
+    temperature, eps) -> scalar float32: L = sum_i w_i l_i, with l_i the dual-clip surrogate of token i
+    and w the seq-mean-token-mean weights (paper's constants delta = 0.2, kappa = 3, clip 20)."""
+
+    @staticmethod
+    def forward(ctx, H_s, W_s, tokens, logp_old, logp_teacher, mask, seg_id, n_ids, temperature=1.0, eps=1e-8):
+        if H_s.dtype != torch.bfloat16 or W_s.dtype != torch.bfloat16:
+            raise TypeError("the surrogate path takes bfloat16 H_s and W_s")
+        H_s, W_s = _contig(H_s, W_s)
+        dev = H_s.device
+        T, d = H_s.shape
+        mask = mask.to(torch.uint8).contiguous()
+        seg_id = seg_id.to(torch.int32).contiguous()
+        tokens = tokens.to(torch.int32).contiguous()
+        logp_old = logp_old.float().contiguous()
+        logp_teacher = logp_teacher.float().contiguous()
+        prob = opd_kl.make_problem(T, d, d, W_s.shape[0], opd_kl.OPD_DTYPE_BF16, float(temperature))
+        ws = opd_kl.allocate_workspace(prob, dev)
+        seq_ws = torch.empty(opd_kl.opd_seq_mean_token_mean_workspace_size(int(n_ids)), dtype=torch.uint8,
+                             device=dev)
+        weights = torch.empty(T, device=dev, dtype=torch.float32)
+        loss_tok = torch.empty(T, device=dev, dtype=torch.float32)
+        logp = torch.empty(T, device=dev, dtype=torch.float32)
+        dH = torch.empty(H_s.shape, device=dev, dtype=torch.float32)
+        dW = torch.empty(W_s.shape, device=dev, dtype=torch.float32)
+        total = torch.empty(1, device=dev, dtype=torch.float32)
+        opd_kl.opd_seq_mean_token_mean_device(seg_id, mask, int(n_ids), float(eps), None, weights, None, seq_ws)
+        opd_kl.opd_surrogate_fwd_bwd(prob, H_s, W_s, tokens, logp_old, logp_teacher, mask, weights, loss_tok, logp,
+                                     dH, dW, False, ws)
+        opd_kl.opd_seq_mean_token_mean_device(seg_id, mask, int(n_ids), float(eps), loss_tok, None, total, seq_ws)
+        ctx.save_for_backward(dH, dW)
+        ctx.dtypes = (H_s.dtype, W_s.dtype)
+        ctx.mark_non_differentiable(tokens, logp_old, logp_teacher, mask, seg_id)
+        return total[0]
+
+    @staticmethod
+    def backward(ctx, grad_loss):
+        dH, dW = ctx.saved_tensors
+        g = grad_loss.float()
+        return (dH * g).to(ctx.dtypes[0]), (dW * g).to(ctx.dtypes[1]), None, None, None, None, None, None, None, None
+
+
+@torch.no_grad()
+def score_tokens(H, W, tokens, mask, temperature=1.0):
+    """(lse, logp) of the given tokens under one head (the frozen teacher's scores): float32 [T] each,
+    zeros on rows with mask 0."""
+    if H.dtype != torch.bfloat16 or W.dtype != torch.bfloat16:
+        raise TypeError("scoring takes bfloat16 H and W")
+    H, W = _contig(H, W)
+    T, d = H.shape
+    prob = opd_kl.make_problem(T, d, d, W.shape[0], opd_kl.OPD_DTYPE_BF16, float(temperature))
+    ws = opd_kl.allocate_workspace(prob, H.device)
+    lse = torch.empty(T, device=H.device, dtype=torch.float32)
+    logp = torch.empty(T, device=H.device, dtype=torch.float32)
+    opd_kl.opd_score_tokens(prob, H, W, tokens.to(torch.int32).contiguous(), mask.to(torch.uint8).contiguous(), lse,
+                            logp, ws)
+    return lse, logp

@@ -69,3 +69,44 @@ def test_seq_mean_loss_autograd(mods, oracle_mod):
     assert abs(float(loss.detach()) - want) <= 1e-4 + 2e-3 * abs(want)
     assert _rel(H_s.grad.float().cpu().numpy(), ref.dH_s) <= 1e-2
     assert _rel(W_s.grad.float().cpu().numpy(), ref.dW_s) <= 1e-2
+
+
+def test_surrogate_loss_autograd_and_scoring(mods, oracle_mod):
+    """OPDSurrogateLoss (device seq-mean-token-mean weights, one surrogate call) and score_tokens
+    against the oracle: the loss, the teacher's scores, and the gradients through .backward()."""
+    ag, lib = mods
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="small", T=500, d_s=128, d_t=192, V=900, tau=1.0,
+                     n_traj=5, traj_len=100, seed=53)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    tok = torch.from_numpy(tokens).cuda()
+    mask = torch.from_numpy(lay.mask).cuda()
+    # the teacher's scores of the sampled tokens, then a behaviour policy near the student
+    lse_t, lp_t = ag.score_tokens(x["H_t"], x["W_t"], tok, mask, w.tau)
+    Ht, Wt = synth.host_values(x["H_t"]), synth.host_values(x["W_t"])
+    sup = lay.mask != 0
+    ref_lse, ref_lp = oracle_mod.score(Ht, Wt, tokens, w.tau, rows=np.flatnonzero(sup))
+    assert np.abs(lse_t.cpu().numpy()[sup] - ref_lse).max() <= 1e-4 + 1e-4 * np.abs(ref_lse).max()
+    assert np.abs(lp_t.cpu().numpy()[sup] - ref_lp).max() <= 1e-4 + 1e-4 * np.abs(ref_lp).max()
+    # both sides get the same inputs, none of them from the GPU: the teacher's log-probabilities
+    # from the oracle, a behaviour policy within 5% of the student (no ratio clip is active)
+    _, lp_teacher = oracle_mod.score(Ht, Wt, tokens, w.tau)
+    lp_teacher = lp_teacher.astype(np.float32)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    _, lp_s = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = (lp_s + np.random.default_rng(53).uniform(-0.05, 0.05, w.T)).astype(np.float32)
+    H_s = x["H_s"].clone().requires_grad_(True)
+    W_s = x["W_s"].clone().requires_grad_(True)
+    n_ids = int(lay.seg_id.max()) + 1
+    loss = ag.OPDSurrogateLoss.apply(H_s, W_s, tok, torch.from_numpy(logp_old).cuda(),
+                                     torch.from_numpy(lp_teacher).cuda(), mask, torch.from_numpy(lay.seg_id).cuda(),
+                                     n_ids, w.tau)
+    (3.0 * loss).backward()
+    wts = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), lp_teacher.astype(np.float64),
+                               lay.mask, 3.0 * wts, w.tau)
+    want = float(np.dot(wts, ref.loss))
+    assert abs(float(loss.detach()) - want) <= 1e-4 + 2e-3 * abs(want)
+    assert _rel(H_s.grad.float().cpu().numpy(), ref.dH_s) <= 1e-2
+    assert _rel(W_s.grad.float().cpu().numpy(), ref.dW_s) <= 1e-2
