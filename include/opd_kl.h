@@ -101,9 +101,19 @@ typedef struct {
  * one call over the whole batch. */
 size_t opd_kl_workspace_size(const opd_problem* problem);
 
+/* Bytes of device workspace that the forward-only calls need: opd_kl_forward and
+ * opd_score_tokens. It is the leading part of the opd_kl_workspace_size layout
+ * (control block, row indices, gathered rows, per-split statistics) without the
+ * backward's row constants, dz buffer and dH_s partial sums, so a forward at the
+ * Qwen3-1.7B shape (T = 16,384, d_s = 2,048, d_t = 4,096, V = 151,936) needs 0.24 GB
+ * instead of 5.36 GB.
+ * A workspace of either size serves those two calls; the backward, fwd_bwd and
+ * surrogate calls need the full size. Returns 0 for an invalid problem. */
+size_t opd_kl_forward_workspace_size(const opd_problem* problem);
+
 /* Forward (Eq. reverse-kl): per-token KL and the per-row statistics the backward
  * needs. kl_out [T] and stats [T, 3] are written for every row (zeros on
- * unsupervised rows). */
+ * unsupervised rows). The workspace needs opd_kl_forward_workspace_size bytes. */
 opd_status opd_kl_forward(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
                           const void* W_t, const uint8_t* mask, float* kl_out, float* stats, void* workspace,
                           size_t workspace_bytes, void* stream);
@@ -152,7 +162,8 @@ opd_status opd_kl_seq_mean_fwd_bwd(const opd_problem* problem, const void* H_s, 
  * student's enters the ratio (Eq. opd-ratio). H [T, d], W [V, d] bf16 with d =
  * problem->d_s (problem->d_t is not used; pass any valid value, e.g. d_s); tokens [T]
  * int32 in [0, V) (an id outside that range sets the workspace status, reported as
- * OPD_ERR_INVALID_ARG by opd_kl_get_status). Workspace as for opd_kl_forward. bf16 only
+ * OPD_ERR_INVALID_ARG by opd_kl_get_status). The workspace needs opd_kl_forward_workspace_size
+ * bytes, as for opd_kl_forward. bf16 only
  * (OPD_ERR_UNSUPPORTED otherwise). */
 opd_status opd_score_tokens(const opd_problem* problem, const void* H, const void* W, const int32_t* tokens,
                             const uint8_t* mask, float* lse_out, float* logp_out, void* workspace,
@@ -204,6 +215,11 @@ opd_status opd_surrogate_fwd_bwd(const opd_problem* problem, const void* H_s, co
  *   - Rows are not compacted: unsupervised rows are computed and then written
  *     as zeros, so the tensor-core work scales with T rather than with the
  *     supervised count.
+ *   - Device-side failures: there is no workspace, so opd_kl_get_status cannot
+ *     report them. If a bounded wait of the call runs out, the call fills every
+ *     kl_out and stats entry with NaN instead. It still returns OPD_OK, because it
+ *     does not synchronise; only with OPD_KL_SYNC_CHECK=1 does it synchronise and
+ *     return OPD_ERR_TIMEOUT (or OPD_ERR_NONFINITE for a non-finite output).
  * Allocates nothing: no cudaMalloc, cudaFree or allocating library call. */
 opd_status opd_kl_forward_noalloc(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,
                                   const void* W_t, const uint8_t* mask, float* kl_out, float* stats, void* stream);

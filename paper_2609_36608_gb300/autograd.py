@@ -17,6 +17,12 @@ log-probabilities (no gradient).
 
 Gradients come back in the dtype of the tensors they belong to (autograd's rule); the
 library computes them in float32.
+
+Errors found on the device (a token id outside [0, V), a response id >= n_ids, a bounded
+wait that ran out) set a status word in the call's workspace; these functions do not read
+it, so outside debug mode such a call returns a wrong loss without raising. With
+OPD_KL_SYNC_CHECK=1 in the environment every library call synchronises, reads that word
+and scans its outputs for NaN and infinity, and the binding raises OpdError.
 """
 
 from __future__ import annotations
@@ -53,14 +59,15 @@ class OPDReverseKL(torch.autograd.Function):
         H_s, H_t, W_s, W_t = _contig(H_s, H_t, W_s, W_t)
         mask = mask.to(torch.uint8).contiguous()
         prob = _problem(H_s, H_t, W_s, W_t, temperature)
-        ws = opd_kl.allocate_workspace(prob, H_s.device)
+        # the forward needs only the leading part of the workspace (no dz buffer); the
+        # backward takes a full one, so the T x V dz memory is held only while it runs
+        ws = opd_kl.allocate_workspace(prob, H_s.device, forward_only=True)
         T = H_s.shape[0]
         kl = torch.empty(T, device=H_s.device, dtype=torch.float32)
         stats = torch.empty(T, 3, device=H_s.device, dtype=torch.float32)
         opd_kl.opd_kl_forward(prob, H_s, H_t, W_s, W_t, mask, kl, stats, ws)
         ctx.save_for_backward(H_s, H_t, W_s, W_t, mask, stats)
         ctx.temperature = float(temperature)
-        ctx.mark_non_differentiable(mask)
         return kl
 
     @staticmethod
@@ -138,7 +145,6 @@ class OPDSurrogateLoss(torch.autograd.Function):
         opd_kl.opd_seq_mean_token_mean_device(seg_id, mask, int(n_ids), float(eps), loss_tok, None, total, seq_ws)
         ctx.save_for_backward(dH, dW)
         ctx.dtypes = (H_s.dtype, W_s.dtype)
-        ctx.mark_non_differentiable(tokens, logp_old, logp_teacher, mask, seg_id)
         return total[0]
 
     @staticmethod
@@ -157,7 +163,7 @@ def score_tokens(H, W, tokens, mask, temperature=1.0):
     H, W = _contig(H, W)
     T, d = H.shape
     prob = opd_kl.make_problem(T, d, d, W.shape[0], opd_kl.OPD_DTYPE_BF16, float(temperature))
-    ws = opd_kl.allocate_workspace(prob, H.device)
+    ws = opd_kl.allocate_workspace(prob, H.device, forward_only=True)
     lse = torch.empty(T, device=H.device, dtype=torch.float32)
     logp = torch.empty(T, device=H.device, dtype=torch.float32)
     opd_kl.opd_score_tokens(prob, H, W, tokens.to(torch.int32).contiguous(), mask.to(torch.uint8).contiguous(), lse,

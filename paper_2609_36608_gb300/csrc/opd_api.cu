@@ -25,10 +25,13 @@ inline size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct WsLayout {
   size_t ctrl = 0, idx = 0, pos = 0, hs_g = 0, ht_g = 0, partials = 0, rowc = 0, dz = 0, dh_g = 0, total = 0;
+  size_t fwd_total = 0;  // the prefix that forward-only calls touch (no backward constants, dz or dH_g)
   int64_t T_pad = 0, Vp = 0;
 };
 
-// Workspace layout, 256-byte aligned sections. Sized for every row supervised.
+// Workspace layout, 256-byte aligned sections. Sized for every row supervised. The
+// sections a forward-only call uses come first, so a forward needs only the prefix
+// [0, fwd_total) and a full workspace serves every call.
 WsLayout ws_layout(const opd_problem& p) {
   WsLayout L;
   L.T_pad = (int64_t)round_up((size_t)(p.T > 0 ? p.T : 1), kRowPad);
@@ -47,10 +50,12 @@ WsLayout ws_layout(const opd_problem& p) {
     L.hs_g = take(2 * Tp * (size_t)p.d_s);
     L.ht_g = take(2 * Tp * (size_t)p.d_t);
     L.partials = take(4 * (size_t)kMaxVSplit * 5 * Tp);
+    L.fwd_total = off;
     L.rowc = take(16 * Tp);
     L.dz = take(2 * Tp * (size_t)L.Vp);
     L.dh_g = take(4 * Tp * (size_t)p.d_s);
   } else {
+    L.fwd_total = off;
     L.dz = take(4 * Tp * (size_t)p.V);
   }
   L.total = off;
@@ -197,6 +202,7 @@ struct Call {
   opd_problem p;
   WsLayout L;
   uint8_t* ws;
+  size_t ws_bytes;
   cudaStream_t s;
   DeviceInfo dev;
   Ctrl* ctrl() const { return reinterpret_cast<Ctrl*>(ws + L.ctrl); }
@@ -213,11 +219,16 @@ opd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? OPD_OK : OPD_E
   } while (0)
 #define OPD_CUDA(expr) OPD_TRY(cuda_status(expr))
 
-opd_status begin_call(Call& c, const opd_problem* problem, void* workspace, size_t ws_bytes, void* stream) {
+// forward_only: the call runs no backward, so the workspace prefix of
+// opd_kl_forward_workspace_size bytes is enough.
+opd_status begin_call(Call& c, const opd_problem* problem, void* workspace, size_t ws_bytes, void* stream,
+                      bool forward_only) {
   OPD_TRY(check_problem(problem));
   c.p = *problem;
   c.L = ws_layout(c.p);
-  if (!workspace || !aligned(workspace, 256) || ws_bytes < c.L.total) return OPD_ERR_INVALID_ARG;
+  if (!workspace || !aligned(workspace, 256) || ws_bytes < (forward_only ? c.L.fwd_total : c.L.total))
+    return OPD_ERR_INVALID_ARG;
+  c.ws_bytes = ws_bytes;
   c.ws = static_cast<uint8_t*>(workspace);
   c.s = static_cast<cudaStream_t>(stream);
   c.dev = device_info();
@@ -245,7 +256,7 @@ opd_status finish_call(const Call& c, const Outputs& out = Outputs()) {
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
   if (env_flag("OPD_KL_SYNC_CHECK")) {
     for (int i = 0; i < out.k; ++i) OPD_CUDA(launch_check_finite(out.p[i], out.n[i], c.ctrl(), c.dev.sm_count, c.s));
-    return opd_kl_get_status(c.ws, c.L.total, c.s);
+    return opd_kl_get_status(c.ws, c.ws_bytes, c.s);
   }
   return OPD_OK;
 }
@@ -443,7 +454,7 @@ opd_status run(const opd_problem* problem, const void* H_s, const void* H_t, con
                float* dH_s, float* dW_s, int accumulate_dW, void* workspace, size_t ws_bytes, void* stream,
                bool do_fwd, bool do_bwd, const SeqLoss* seq = nullptr) {
   Call c;
-  OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream));
+  OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream, !do_bwd));
   OPD_TRY(check_inputs(c, H_s, H_t, W_s, W_t, mask));
   const int64_t T = c.p.T;
   if (do_fwd && T > 0 && (!kl_out || !stats_out)) return OPD_ERR_INVALID_ARG;
@@ -510,7 +521,7 @@ opd_status head_call(const opd_problem* problem, const void* H, const void* W, c
                      float* loss_out, float* dH, float* dW, int accumulate_dW, void* workspace, size_t ws_bytes,
                      void* stream, bool surrogate) {
   Call c;
-  OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream));
+  OPD_TRY(begin_call(c, problem, workspace, ws_bytes, stream, !surrogate));
   if (c.p.dtype != OPD_DTYPE_BF16) return OPD_ERR_UNSUPPORTED;
   const int64_t T = c.p.T;
   if (!W || !aligned(W, 16) || !aligned(H, 16)) return OPD_ERR_INVALID_ARG;
@@ -590,6 +601,12 @@ size_t opd_kl_workspace_size(const opd_problem* problem) {
   const opd_status st = check_problem(problem);
   if (st != OPD_OK) return 0;
   return ws_layout(*problem).total;
+}
+
+size_t opd_kl_forward_workspace_size(const opd_problem* problem) {
+  if (!problem) return 0;
+  if (check_problem(problem) != OPD_OK) return 0;
+  return ws_layout(*problem).fwd_total;
 }
 
 opd_status opd_kl_forward(const opd_problem* problem, const void* H_s, const void* H_t, const void* W_s,

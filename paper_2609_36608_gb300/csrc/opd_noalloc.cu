@@ -54,6 +54,22 @@ __global__ void k_noalloc_rows(const uint8_t* __restrict__ mask, int32_t T) {
   if (threadIdx.x < 4) ctrl->work[threadIdx.x] = 0;
 }
 
+// After the combine: if a bounded wait of this call ran out, every kl_out and stats
+// entry becomes NaN, so that a caller who does not synchronise still cannot mistake
+// partial statistics for a result (this entry point has no workspace whose status
+// word the caller could read).
+__global__ void k_noalloc_poison_on_timeout(float* kl_out, float* stats, int32_t T) {
+  const Ctrl* ctrl = reinterpret_cast<const Ctrl*>(g_noalloc_scratch);
+  if ((ctrl->status & kDevTimeout) == 0u) return;
+  const float nan = __int_as_float(0x7fc00000);
+  for (int i = threadIdx.x; i < T; i += blockDim.x) {
+    kl_out[i] = nan;
+    stats[3 * i] = nan;
+    stats[3 * i + 1] = nan;
+    stats[3 * i + 2] = nan;
+  }
+}
+
 // Device address of the scratch array, looked up once per device (with that
 // device current) and cached; host code must not use the symbol itself.
 unsigned char* scratch_address(int dev) {
@@ -157,6 +173,8 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
   if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
     return OPD_ERR_CUDA;
+  k_noalloc_poison_on_timeout<<<1, 1024, 0, s>>>(kl_out, stats, T);
+  if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
 
   const char* sync = std::getenv("OPD_KL_SYNC_CHECK");
   if (sync && sync[0] && sync[0] != '0') {

@@ -58,6 +58,7 @@ def _load() -> ctypes.CDLL:
     vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t
     sig = {
         "opd_kl_workspace_size": (sz, [P]),
+        "opd_kl_forward_workspace_size": (sz, [P]),
         "opd_kl_forward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]),
         "opd_kl_forward_noalloc": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp]),
         "opd_kl_backward": (i32, [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, i32, vp, sz, vp]),
@@ -175,8 +176,14 @@ def opd_kl_workspace_size(problem: opd_problem) -> int:
     return int(_lib.opd_kl_workspace_size(ctypes.byref(problem)))
 
 
-def allocate_workspace(problem: opd_problem, device="cuda") -> torch.Tensor:
-    n = opd_kl_workspace_size(problem)
+def opd_kl_forward_workspace_size(problem: opd_problem) -> int:
+    return int(_lib.opd_kl_forward_workspace_size(ctypes.byref(problem)))
+
+
+def allocate_workspace(problem: opd_problem, device="cuda", forward_only: bool = False) -> torch.Tensor:
+    """A workspace for every call on this problem, or (forward_only) the smaller one that
+    opd_kl_forward and opd_score_tokens need."""
+    n = opd_kl_forward_workspace_size(problem) if forward_only else opd_kl_workspace_size(problem)
     if n == 0:
         raise ValueError("invalid problem")
     return torch.empty(n, dtype=torch.uint8, device=device)

@@ -54,6 +54,36 @@ def test_workspace_size(lib):
         assert lib.opd_kl_workspace_size(bad) == 0
 
 
+def test_forward_workspace_is_the_leading_part_without_dz(lib):
+    for T, ds, dt, V, dtype in ((16384, 2048, 4096, 151936, lib.OPD_DTYPE_BF16), (300, 64, 128, 1000, lib.OPD_DTYPE_BF16),
+                                (64, 64, 128, 1000, lib.OPD_DTYPE_F32)):
+        p = lib.make_problem(T, ds, dt, V, dtype, 1.0)
+        full, fwd = lib.opd_kl_workspace_size(p), lib.opd_kl_forward_workspace_size(p)
+        elem = 2 if dtype == lib.OPD_DTYPE_BF16 else 4
+        assert 0 < fwd and fwd + T * V * elem <= full  # no dz buffer in the forward's part
+        assert fwd % 256 == 0
+    p = lib.make_problem(16384, 2048, 4096, 151936, lib.OPD_DTYPE_BF16, 1.0)
+    assert lib.opd_kl_forward_workspace_size(p) < 0.25e9  # the gathered rows and statistics
+    assert lib.opd_kl_forward_workspace_size(lib.make_problem(8, 12, 8, 8)) == 0
+    # forward-only calls accept the smaller workspace (the call then stops at the missing GPU, or
+    # runs); one byte less, and any backward with it, are rejected before any CUDA call
+    vp = ctypes.c_void_p
+    fake = vp(1 << 20)
+    small = lib.make_problem(300, 64, 128, 1000, lib.OPD_DTYPE_BF16, 1.0)
+    n = lib.opd_kl_forward_workspace_size(small)
+    fwd = lambda nbytes: lib.call_raw("opd_kl_forward", ctypes.byref(small), fake, fake, fake, fake, fake, fake,
+                                      fake, fake, ctypes.c_size_t(nbytes), None)
+    assert fwd(n - 1) == lib.OPD_ERR_INVALID_ARG
+    assert fwd(n) != lib.OPD_ERR_INVALID_ARG
+    score = lambda nbytes: lib.call_raw("opd_score_tokens", ctypes.byref(small), fake, fake, fake, fake, fake,
+                                        fake, fake, ctypes.c_size_t(nbytes), None)
+    assert score(n - 1) == lib.OPD_ERR_INVALID_ARG
+    assert score(n) != lib.OPD_ERR_INVALID_ARG
+    rc = lib.call_raw("opd_kl_backward", ctypes.byref(small), fake, fake, fake, fake, fake, fake, fake, fake, fake,
+                      0, fake, ctypes.c_size_t(n), None)
+    assert rc == lib.OPD_ERR_INVALID_ARG
+
+
 def test_invalid_arguments_rejected_before_any_launch(lib):
     vp = ctypes.c_void_p
     fake = vp(1 << 20)  # never dereferenced: validation fails first

@@ -161,6 +161,71 @@ def test_surrogate_and_scoring_below_one_tile(lib, oracle_mod, shape, tiling):
     assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
 
 
+def test_surrogate_log_ratio_clip_branch(lib, oracle_mod, tiling):
+    """Tokens whose log-ratio r = logp - logp_old lies beyond the +-20 clip (Appendix B.4,
+    Eq. opd-ratio), with both signs of the advantage, beside unclipped tokens.
+
+    Five classes of supervised token, by row: r in [20.5, 40], r in [-40, -20.5], r in
+    [100, 200] (exp(r) overflows fp32 unless r is clipped first), r in [-200, -100], and
+    r in [-0.6, 1.4] off the ratio-clip kinks. Every r keeps at least 0.5 from +-20, far
+    beyond the ~1e-5 difference between the GPU's and the oracle's log-probabilities, so
+    both sides take the same branch. Beyond the clip the ratio is constant, so those
+    tokens must carry no gradient at all: their dH_s rows are exactly zero. With A < 0 and
+    r > 20 the dual clip caps the loss at -kappa A; with A < 0 and r < -20 the loss is
+    -(1 - delta) A. A second call with every supervised token beyond the clip must give
+    dH_s = 0 and dW_s = 0 exactly (a slope kept at r < -20 would leave ~1e-9 there)."""
+    w = _case(T=600, d_s=192, V=1237, tau=0.9, n_traj=6, seed=35)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    _, lp_ref = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    rng = np.random.default_rng(35)
+    cls = np.arange(w.T) % 5
+    r = np.select([cls == 0, cls == 1, cls == 2, cls == 3],
+                  [rng.uniform(20.5, 40, w.T), -rng.uniform(20.5, 40, w.T), rng.uniform(100, 200, w.T),
+                   -rng.uniform(100, 200, w.T)], _clear_offsets(36, w.T))
+    # both signs of A in every class: the sign alternates every five rows
+    sign = np.where((np.arange(w.T) // 5) % 2 == 0, 1.0, -1.0)
+    adv = sign * rng.uniform(0.2, 1.5, w.T)
+    sup = lay.mask != 0
+    clipped = sup & (cls != 4)
+    for c in range(5):
+        for sgn in (1.0, -1.0):
+            assert (sup & (cls == c) & (sign == sgn)).any(), (c, sgn)
+    weights = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask).astype(np.float32)
+    for everything_clipped in (False, True):
+        rr = np.where(cls == 4, 30.0 * sign, r) if everything_clipped else r
+        logp_old = (lp_ref - rr).astype(np.float32)
+        logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
+        r32 = lp_ref - logp_old.astype(np.float64)  # the log-ratio after the fp32 rounding of logp_old
+        far = np.abs(np.abs(r32) - 20.0) >= 0.5
+        assert far[sup].all()
+        loss, lp, dH, dW = _surrogate(lib, w, x, tokens, logp_old, logp_teacher, lay.mask, weights)
+        ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                                   lay.mask, weights.astype(np.float64), w.tau)
+        assert np.isfinite(loss).all() and np.isfinite(dH).all() and np.isfinite(dW).all()
+        _close(lp[sup], ref.logp_s[sup], 1e-4, 1e-4, "logp")
+        _close(loss, ref.loss, 1e-4, 2e-3, "loss")
+        A = logp_teacher.astype(np.float64) - logp_old.astype(np.float64)
+        hi, lo = sup & (r32 > 20), sup & (r32 < -20)
+        _close(loss[hi & (A < 0)], -oracle_mod.KAPPA * A[hi & (A < 0)], 1e-4, 2e-3, "dual clip, r > 20")
+        _close(loss[hi & (A > 0)], -(1 + oracle_mod.DELTA) * A[hi & (A > 0)], 1e-4, 2e-3, "ratio clip, r > 20")
+        _close(loss[lo & (A < 0)], -(1 - oracle_mod.DELTA) * A[lo & (A < 0)], 1e-4, 2e-3, "ratio clip, r < -20")
+        _close(loss[lo & (A > 0)], np.zeros(int((lo & (A > 0)).sum())), 1e-4, 0, "r < -20, A > 0")
+        rows_clipped = sup & (np.abs(r32) > 20)
+        assert (dH[rows_clipped] == 0).all() and (ref.dH_s[rows_clipped] == 0).all()
+        assert (dH[~sup] == 0).all() and (loss[~sup] == 0).all()
+        if everything_clipped:
+            assert rows_clipped[sup].all()
+            assert (dH == 0).all() and (dW == 0).all()
+            assert (ref.dW_s == 0).all()
+        else:
+            assert clipped.sum() > 0 and (sup & ~clipped).sum() > 0
+            assert _rel(dH, ref.dH_s) <= 1e-2, _rel(dH, ref.dH_s)
+            assert _rel(dW, ref.dW_s) <= 1e-2, _rel(dW, ref.dW_s)
+
+
 def _random_cases(n, seed=4049):
     rng = np.random.default_rng(seed)
     return [dict(T=int(rng.integers(1, 600)), d_s=8 * int(rng.integers(1, 41)), V=int(rng.integers(2, 5000)),

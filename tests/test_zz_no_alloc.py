@@ -1,13 +1,13 @@
-"""The workspace-free forward entry point against the regular forward.
+"""The workspace-free forward entry point against the oracle and the regular forward.
 
 opd_kl_forward_noalloc serves callers that may not allocate device memory at
 all, such as a host process that owns the whole GPU through its own fixed pool
 and forbids libraries from calling cudaMalloc. It keeps its scratch in a fixed
 array inside the library instead of a caller-provided workspace. This file
-checks it through the C ABI against opd_kl_forward, with the same tolerance as
-the parity tests, on three calls in a row with different problems (each call
-reuses the array the previous one left behind). It runs last so that a
-failure here leaves every other test already run.
+checks it through the C ABI against the float64 oracle and against
+opd_kl_forward, with the same tolerance as the parity tests, on three calls in a
+row with different problems (each call reuses the array the previous one left
+behind). It runs last so that a failure here leaves every other test already run.
 """
 
 import numpy as np
@@ -53,7 +53,7 @@ def _both(lib, w):
     return lay.mask != 0, kl.cpu().numpy(), st.cpu().numpy(), kl_ref.cpu().numpy(), st_ref.cpu().numpy()
 
 
-def test_noalloc_forward_matches_workspace_forward_on_three_calls(lib):
+def test_noalloc_forward_matches_oracle_and_workspace_forward_on_three_calls(lib, oracle_mod):
     # every row is scheduled here (no compaction): T = 300 leaves a last row tile of 44 rows,
     # which runs at half height on a CTA pair
     cases = [_case("noalloc_a", T=700, seed=21),
@@ -62,6 +62,17 @@ def test_noalloc_forward_matches_workspace_forward_on_three_calls(lib):
              _case("noalloc_c", T=300, d_s=192, d_t=256, V=3000, tau=1.3, seed=23, traj_len=300)]
     for w in cases:
         sup, kl, st, kl_ref, st_ref = _both(lib, w)
+        # against the float64 oracle, on every supervised row
+        x = synth.hidden_and_heads(w, "cuda")
+        rows = np.flatnonzero(sup)
+        ref = oracle_mod.opd_kl(*(synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")), sup,
+                                np.zeros(w.T), w.tau, rows=rows, want_dH=False, want_dW=False)
+        excess = np.abs(kl[rows] - ref.kl) - (KL_ABS + KL_REL * np.abs(ref.kl))
+        assert excess.max() <= 0, (w.name, "oracle", float(excess.max()))
+        for col, want in ((0, ref.lse_s), (1, ref.lse_t), (2, ref.kl)):
+            tol = 1e-4 + (KL_REL if col == 2 else 1e-5) * np.abs(want)
+            assert (np.abs(st[rows, col] - want) <= tol).all(), (w.name, "stats column", col)
+        # against the workspace forward
         excess = np.abs(kl - kl_ref) - (KL_ABS + KL_REL * np.abs(kl_ref))
         assert excess.max() <= 0, (w.name, float(excess.max()))
         assert (kl[~sup] == 0).all() and (st[~sup] == 0).all()
