@@ -572,11 +572,16 @@ def run_gpu(args):
 
     e2e_steps(1)
     barrier(world)
+    sampler_e2e = ClockSampler(local) if rank == 0 else None
+    if sampler_e2e:
+        sampler_e2e.start()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record()
     e2e_steps(args.steps)
     e1.record()
     torch.cuda.synchronize()
+    if sampler_e2e:
+        sampler_e2e.stop()
     barrier(world)
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     e2e_value = whole_job_rate(R, args.steps, world, e2e_ms)
@@ -626,7 +631,8 @@ def run_gpu(args):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "parity_sampled_rows": parity,
-        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_ms / args.steps, "clocks": sampler_e2e.summary() if sampler_e2e else None},
         # launches in the timed region: the per-kernel pass runs the same K steps
         "gpu_launches": int(sum(v["launches"] for v in kernels.values())),
         "clocks": clocks,

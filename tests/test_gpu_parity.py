@@ -91,6 +91,49 @@ def _full_check(lib, oracle_mod, w, mask=None, g=None, tight=False, **kw):
     return out, ref, x
 
 
+@pytest.mark.parametrize("which", ["tiny_fp32", "bf16"])
+def test_forward_and_scoring_with_the_forward_only_workspace(lib, oracle_mod, which):
+    """opd_kl_forward and opd_score_tokens given exactly opd_kl_forward_workspace_size bytes (no dz
+    buffer) match the oracle, and write nothing past those bytes: a sentinel tail behind the
+    workspace view stays intact."""
+    w = synth.WORKLOADS["tiny_fp32"] if which == "tiny_fp32" else _small_bf16(T=600, seed=12)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    dtype = lib.OPD_DTYPE_F32 if w.dtype == "f32" else lib.OPD_DTYPE_BF16
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
+    n = lib.opd_kl_forward_workspace_size(prob)
+    assert 0 < n < lib.opd_kl_workspace_size(prob)
+    buf = torch.full((n + 4096,), 0xA5, dtype=torch.uint8, device="cuda")
+    ws = buf[:n]
+    mask = torch.from_numpy(lay.mask).cuda()
+    kl = torch.full((w.T,), float("nan"), device="cuda")
+    stats = torch.full((w.T, 3), float("nan"), device="cuda")
+    lib.opd_kl_forward(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, kl, stats, ws)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+    sup = lay.mask != 0
+    ref = oracle_mod.opd_kl(*_host(x), lay.mask, np.zeros(w.T), w.tau, want_dH=False, want_dW=False)
+    _check_kl(kl.cpu().numpy(), ref.kl)
+    st = stats.cpu().numpy()
+    np.testing.assert_allclose(st[sup, 0], ref.lse_s[sup], rtol=1e-5, atol=1e-4)
+    np.testing.assert_allclose(st[sup, 1], ref.lse_t[sup], rtol=1e-5, atol=1e-4)
+    if dtype == lib.OPD_DTYPE_BF16:  # token scoring (bf16 only) with the same workspace
+        tokens = synth.token_ids(w.seed, w.T, w.V)
+        sprob = lib.make_problem(w.T, w.d_t, w.d_t, w.V, dtype, w.tau)
+        m = lib.opd_kl_forward_workspace_size(sprob)
+        sws = buf[:m] if m <= n else torch.empty(m, dtype=torch.uint8, device="cuda")
+        lse = torch.full((w.T,), float("nan"), device="cuda")
+        lp = torch.full((w.T,), float("nan"), device="cuda")
+        lib.opd_score_tokens(sprob, x["H_t"], x["W_t"], torch.from_numpy(tokens).cuda(), mask, lse, lp, sws)
+        torch.cuda.synchronize()
+        assert lib.opd_kl_get_status(sws) == lib.OPD_OK
+        ref_lse, ref_lp = oracle_mod.score(synth.host_values(x["H_t"]), synth.host_values(x["W_t"]), tokens, w.tau,
+                                           rows=np.flatnonzero(sup))
+        np.testing.assert_allclose(lse.cpu().numpy()[sup], ref_lse, rtol=1e-4, atol=1e-4)
+        np.testing.assert_allclose(lp.cpu().numpy()[sup], ref_lp, rtol=1e-4, atol=1e-4)
+    assert (buf[n:] == 0xA5).all()
+
+
 @pytest.mark.parametrize("layout", ["tiny", "tiny_alt"])
 def test_tiny_fp32_config(lib, oracle_mod, layout):
     w = synth.scaled(synth.WORKLOADS["tiny_fp32"], layout=layout)
