@@ -176,6 +176,20 @@ def whole_job_rate(units_per_rank_step: int, steps: int, world: int, max_ms: flo
     return units_per_rank_step * steps * world / (max_ms / 1000.0)
 
 
+def sum_over_ranks(x: int, world: int, device) -> int:
+    if world == 1:
+        return int(x)
+    t = torch.tensor([int(x)], dtype=torch.int64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.SUM)
+    return int(t.item())
+
+
+def rank_workload(w, rank: int):
+    """Each rank's own batch under data parallelism: rank 0 keeps the workload's seed (its
+    batch is the single-GPU batch), rank k draws another packed batch of the same shape."""
+    return w if rank == 0 else synth.scaled(w, seed=w.seed + 1000 * rank)
+
+
 # -------------------------------------------------------------------- flops
 
 def step_flops(w, R):
@@ -303,13 +317,30 @@ PATH_METRICS = {
 }
 
 
-def path_setup(path, w, lay, x, dev, opd_kl):
+def path_setup(path, w, lay, x, dev, opd_kl, world=1, rank=0):
     """Per-step device inputs (the tensors the e2e leg copies from the host each step), the
     step function over them, the output read back each step, and the step's FLOPs."""
     R = int(lay.mask.sum())
     mask = torch.from_numpy(lay.mask).to(dev)
     weights = torch.from_numpy(opd_kl.opd_seq_mean_token_mean_weights(lay.seg_id, lay.mask, 1e-8)).to(dev)
     dtype = opd_kl.OPD_DTYPE_BF16 if w.dtype == "bf16" else opd_kl.OPD_DTYPE_F32
+    if path == "kl" and world > 1:
+        # token-sharded data parallelism: this rank's batch, the paper's batch loss over every
+        # rank's rows (response ids made global), dW_s and L summed over the ranks each step
+        from paper_2609_36608_gb300 import data_parallel
+        n_local = int(lay.seg_id.max()) + 1
+        n_max = int(max_over_ranks(float(n_local), world, dev))
+        seg = np.where(lay.seg_id >= 0, lay.seg_id + rank * n_max, -1).astype(np.int32)
+        sharded = data_parallel.ShardedSeqMeanKL(w.T, w.d_s, w.d_t, w.V, n_max * world, w.tau, device=dev,
+                                                 dtype=dtype)
+        dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+        inputs = {"H_s": x["H_s"], "H_t": x["H_t"], "mask": mask, "seg_id": torch.from_numpy(seg).to(dev)}
+
+        def step(i):
+            sharded.step(i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["seg_id"], dH, dW)
+        step.outputs = {"kl": sharded.kl, "dH": dH}
+        executed, algorithmic = step_flops(w, R)
+        return inputs, step, sharded.loss, sharded.ws, executed, algorithmic
     if path == "kl":
         prob = opd_kl.make_problem(w.T, w.d_s, w.d_t, w.V, dtype, w.tau)
         ws = opd_kl.allocate_workspace(prob, dev)
@@ -484,11 +515,12 @@ def run_gpu(args):
     build.build()
     from paper_2609_36608_gb300 import opd_kl
 
-    w = synth.WORKLOADS[args.workload]
+    w = rank_workload(synth.WORKLOADS[args.workload], rank)
     lay = synth.layout(w)
     R = int(lay.mask.sum())
+    R_job = sum_over_ranks(R, world, dev)  # supervised rows of all ranks' batches per step
     x = synth.hidden_and_heads(w, dev)
-    inputs, step, result, ws, executed, algorithmic = path_setup(args.path, w, lay, x, dev, opd_kl)
+    inputs, step, result, ws, executed, algorithmic = path_setup(args.path, w, lay, x, dev, opd_kl, world, rank)
 
     sampler = ClockSampler(local) if rank == 0 else None
     if sampler:
@@ -517,7 +549,7 @@ def run_gpu(args):
         raise RuntimeError("device status after the timed region is not OK")
     ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_step = ms / args.steps
-    value = whole_job_rate(R, args.steps, world, ms)
+    value = whole_job_rate(R_job, args.steps, 1, ms)
     clocks = sampler.summary() if sampler else None  # samples of the timed region only
 
     # per-kernel times for the roofline: a second pass of the same K steps with every
@@ -584,7 +616,7 @@ def run_gpu(args):
         sampler_e2e.stop()
     barrier(world)
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-    e2e_value = whole_job_rate(R, args.steps, world, e2e_ms)
+    e2e_value = whole_job_rate(R_job, args.steps, 1, e2e_ms)
 
     if rank != 0:
         torch.distributed.destroy_process_group() if world > 1 else None
@@ -622,8 +654,11 @@ def run_gpu(args):
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded counter-based generator, packed multi-turn layout with masked observations "
                 "and inserted tokens",
-        "config": {"workload": w.name, "T": w.T, "R": R, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
-                   "temperature": w.tau, "parallelism": "replicas" if world > 1 else "single",
+        "config": {"workload": w.name, "T": w.T, "R": R, "R_all_ranks": R_job, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
+                   "temperature": w.tau,
+                   "parallelism": (f"dp{world}: token-sharded, one {w.T}-token batch per GPU, dW_s and the "
+                                   "loss all-reduced each step" if world > 1 and args.path == "kl" else
+                                   "replicas" if world > 1 else "single"),
                    "l2": "inputs larger than L2 (W_s + W_t = %.2f GB)" % ((w.d_s + w.d_t) * w.V * 2 / 1e9)},
         "tflops_executed": executed / (ms_step / 1000.0) / 1e12,
         "tflops_algorithmic": algorithmic / (ms_step / 1000.0) / 1e12,

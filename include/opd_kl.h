@@ -247,6 +247,31 @@ opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* 
                                           float eps, const float* loss_in, float* w_out, float* loss_out,
                                           void* workspace, size_t workspace_bytes, void* stream);
 
+/* The same weights for a batch whose rows are spread over several processes (token-sharded
+ * data parallelism: each process holds some rows of the batch; a response may even straddle
+ * two processes). The paper's L is over the whole batch (Appendix B.4, Eq. opd-surrogate),
+ * so n_b and |B| must count every process's rows. Two calls per process, with one sum over
+ * processes between them:
+ *   1. opd_seq_mean_token_mean_counts writes counts [2, n_ids] int32 (device): row b of the
+ *      first plane is the number of this process's supervised rows of response b, of the
+ *      second plane the number of all its rows of response b. An id >= n_ids is skipped and
+ *      sets the workspace status (OPD_ERR_INVALID_ARG from opd_kl_get_status).
+ *   2. The caller sums counts over the processes (an all-reduce of 2 n_ids int32 values).
+ *   3. opd_seq_mean_token_mean_from_counts takes the summed counts and writes this process's
+ *      weights w_out [T] (may be NULL) and, when loss_in [T] and loss_out [1] are given,
+ *      loss_out[0] = sum over this process's rows of w_i loss_in[i] (in double, in no fixed
+ *      order). The sum of loss_out over the processes is the batch loss L.
+ * Response ids are global ids in [0, n_ids) (ids < 0 mark rows outside every response).
+ * With one process the result equals opd_seq_mean_token_mean_device. Workspaces as for
+ * opd_seq_mean_token_mean_device (the status word of step 1 stays set through step 3).
+ * seg_id, mask, counts, loss_in, w_out and loss_out are device memory. */
+opd_status opd_seq_mean_token_mean_counts(const int32_t* seg_id, const uint8_t* mask, int64_t T, int64_t n_ids,
+                                          int32_t* counts, void* workspace, size_t workspace_bytes, void* stream);
+opd_status opd_seq_mean_token_mean_from_counts(const int32_t* seg_id, const uint8_t* mask, int64_t T, int64_t n_ids,
+                                               const int32_t* counts, float eps, const float* loss_in,
+                                               float* w_out, float* loss_out, void* workspace,
+                                               size_t workspace_bytes, void* stream);
+
 /* Reads and clears the device status word in the workspace, after
  * synchronising the stream: OPD_OK, OPD_ERR_TIMEOUT if a bounded wait in the last
  * call ran out, or OPD_ERR_INVALID_ARG if a token id was outside [0, V) (or a response

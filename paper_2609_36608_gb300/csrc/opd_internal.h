@@ -130,6 +130,16 @@ cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, 
                                        const float* loss_in, float* w_out, float* loss_out, Ctrl* ctrl,
                                        bool clear_status, void* scratch, int n_sm, cudaStream_t s);
 cudaError_t launch_store_loss(const double* acc, float* loss_out, cudaStream_t s);
+// The histogram pass alone, into counts [2, n_ids] (supervised rows, then all rows, per id);
+// clears ctrl->status first, and bad ids set it.
+cudaError_t launch_seq_counts(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, int32_t* counts,
+                              Ctrl* ctrl, int n_sm, cudaStream_t s);
+// Weights (and sum_i w_i loss_in[i]) from a histogram summed over processes (ctrl->status is
+// left as the histogram pass set it); scratch holds
+// the double accumulator and |B| (seq_mean_token_mean_scratch_bytes(0) bytes suffice).
+cudaError_t launch_seq_from_counts(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids,
+                                   const int32_t* counts, float eps, const float* loss_in, float* w_out,
+                                   float* loss_out, Ctrl* ctrl, void* scratch, int n_sm, cudaStream_t s);
 // C = A * B^T with A [M, K] and B [N, K] given through tensor maps; a_mn / b_mn select
 // MN-major operand tiles (the operand's contiguous dimension is M or N, not K).
 cudaError_t launch_gemm(bool a_mn, bool b_mn, const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,

@@ -5,6 +5,11 @@
 // including responses whose tokens are all masked). Three small memory-bound passes:
 // a histogram of supervised tokens per response id, the count of distinct ids, then the
 // weights and (optionally) sum_i w_i l_i.
+//
+// For a batch whose rows are spread over several processes the histogram is its own
+// pass (launch_seq_counts: supervised rows and all rows per id, summable across
+// processes), and the last two passes run from the summed histogram
+// (launch_seq_from_counts), so every process gets the whole batch's n_b and |B|.
 #include "opd_device.cuh"
 #include "opd_internal.h"
 
@@ -27,8 +32,15 @@ __global__ void k_seq_zero(uint32_t* status, bool clear_status, int32_t* counts,
   }
 }
 
+__global__ void k_seq_zero_counts(uint32_t* status, int32_t* counts, int32_t n) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) counts[i] = 0;
+  if (blockIdx.x == 0 && threadIdx.x == 0) *status = 0u;
+}
+
+// counts[b] += supervised rows of response b; present[b] = 1 (or, with count_rows, += every
+// row of b, so that the planes of several processes can be summed).
 __global__ void k_seq_hist(const int32_t* __restrict__ seg, const uint8_t* __restrict__ mask, int32_t T,
-                           int32_t n_ids, int32_t* counts, int32_t* present, uint32_t* status) {
+                           int32_t n_ids, int32_t* counts, int32_t* present, uint32_t* status, bool count_rows) {
   for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
     const int b = seg[i];
     if (b < 0) continue;
@@ -36,14 +48,19 @@ __global__ void k_seq_hist(const int32_t* __restrict__ seg, const uint8_t* __res
       atomicOr(status, kDevBadToken);
       continue;
     }
-    present[b] = 1;
+    if (count_rows)
+      atomicAdd(&present[b], 1);
+    else
+      present[b] = 1;
     if (mask[i]) atomicAdd(&counts[b], 1);
   }
 }
 
+// |B|: the ids with at least one row (present[] may hold row counts summed over processes).
 __global__ void k_seq_count(const int32_t* __restrict__ present, int32_t n_ids, int32_t* n_resp) {
   int local = 0;
-  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_ids; i += gridDim.x * blockDim.x) local += present[i];
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_ids; i += gridDim.x * blockDim.x)
+    local += present[i] != 0 ? 1 : 0;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) local += __shfl_xor_sync(0xffffffffu, local, o);
   if ((threadIdx.x & 31) == 0 && local) atomicAdd(n_resp, local);
@@ -77,10 +94,6 @@ cudaError_t launch_store_loss(const double* acc, float* loss_out, cudaStream_t s
   return cudaGetLastError();
 }
 
-namespace {
-
-}  // namespace
-
 size_t seq_mean_token_mean_scratch_bytes(int64_t n_ids) { return 16 + 8 * (size_t)n_ids; }
 
 double* seq_mean_token_mean_acc(void* scratch) { return static_cast<double*>(scratch); }
@@ -100,8 +113,40 @@ cudaError_t launch_seq_mean_token_mean(const int32_t* seg, const uint8_t* mask, 
     return (int)(b < 1 ? 1 : b);
   };
   k_seq_zero<<<blocks(n_ids), threads, 0, s>>>(status, clear_status, counts, present, n_ids, n_resp, acc);
-  k_seq_hist<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, present, status);
+  k_seq_hist<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, present, status, false);
   k_seq_count<<<blocks(n_ids), threads, 0, s>>>(present, n_ids, n_resp);
+  k_seq_weights<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, n_resp, eps, loss_in, w_out, acc);
+  if (loss_out) k_seq_store<<<1, 1, 0, s>>>(acc, loss_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_counts(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids, int32_t* counts,
+                              Ctrl* ctrl, int n_sm, cudaStream_t s) {
+  const int threads = 256;
+  auto blocks = [&](long work) {
+    long b = (work + threads - 1) / threads;
+    if (b > (long)n_sm * 4) b = (long)n_sm * 4;
+    return (int)(b < 1 ? 1 : b);
+  };
+  // counts [2, n_ids]: supervised rows, then all rows, of each response id
+  k_seq_zero_counts<<<blocks(2 * (long)n_ids), threads, 0, s>>>(&ctrl->status, counts, 2 * n_ids);
+  k_seq_hist<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, counts + n_ids, &ctrl->status, true);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_from_counts(const int32_t* seg, const uint8_t* mask, int32_t T, int32_t n_ids,
+                                   const int32_t* counts, float eps, const float* loss_in, float* w_out,
+                                   float* loss_out, Ctrl* ctrl, void* scratch, int n_sm, cudaStream_t s) {
+  double* acc = static_cast<double*>(scratch);
+  int32_t* n_resp = reinterpret_cast<int32_t*>(acc + 1);
+  const int threads = 256;
+  auto blocks = [&](long work) {
+    long b = (work + threads - 1) / threads;
+    if (b > (long)n_sm * 4) b = (long)n_sm * 4;
+    return (int)(b < 1 ? 1 : b);
+  };
+  k_seq_zero<<<1, threads, 0, s>>>(&ctrl->status, false, nullptr, nullptr, 0, n_resp, acc);
+  k_seq_count<<<blocks(n_ids), threads, 0, s>>>(counts + n_ids, n_ids, n_resp);
   k_seq_weights<<<blocks(T), threads, 0, s>>>(seg, mask, T, n_ids, counts, n_resp, eps, loss_in, w_out, acc);
   if (loss_out) k_seq_store<<<1, 1, 0, s>>>(acc, loss_out);
   return cudaGetLastError();

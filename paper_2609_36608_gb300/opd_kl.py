@@ -75,6 +75,9 @@ def _load() -> ctypes.CDLL:
         "opd_kl_seq_mean_fwd_bwd": (i32, [P, vp, vp, vp, vp, vp, vp, i64, ctypes.c_float, vp, vp, vp, vp, vp, i32,
                                           vp, sz, vp]),
         "opd_seq_mean_token_mean_device": (i32, [vp, vp, i64, i64, ctypes.c_float, vp, vp, vp, vp, sz, vp]),
+        "opd_seq_mean_token_mean_counts": (i32, [vp, vp, i64, i64, vp, vp, sz, vp]),
+        "opd_seq_mean_token_mean_from_counts": (i32, [vp, vp, i64, i64, vp, ctypes.c_float, vp, vp, vp, vp, sz,
+                                                      vp]),
         "opd_kl_profile_start": (i32, []),
         "opd_kl_profile_stop": (i32, [ctypes.POINTER(opd_kernel_time), i32, ctypes.POINTER(i32)]),
     }
@@ -299,6 +302,26 @@ def opd_seq_mean_token_mean_device(seg_id, mask, n_ids: int, eps: float = 1e-8, 
             b(workspace, "workspace"), _nbytes(workspace)]
     _check(_call("opd_seq_mean_token_mean_device", b, args, stream), "opd_seq_mean_token_mean_device")
     return workspace
+
+
+def opd_seq_mean_token_mean_counts(seg_id, mask, n_ids: int, counts, workspace, stream=None) -> None:
+    """This process's rows per response id: counts [2, n_ids] int32 (supervised rows, all rows)."""
+    T, b = seg_id.numel(), _Buffers()
+    args = [b(seg_id, "seg_id", _I32, T), b(mask, "mask", _BYTE, T), T, int(n_ids),
+            b(counts, "counts", _I32, 2 * int(n_ids)), b(workspace, "workspace"), _nbytes(workspace)]
+    _check(_call("opd_seq_mean_token_mean_counts", b, args, stream), "opd_seq_mean_token_mean_counts")
+
+
+def opd_seq_mean_token_mean_from_counts(seg_id, mask, n_ids: int, counts, eps: float = 1e-8, loss_in=None,
+                                        w_out=None, loss_out=None, workspace=None, stream=None) -> None:
+    """seq-mean-token-mean weights of this process's rows (and its part of the batch loss) from
+    the per-id counts summed over every process."""
+    T, b = seg_id.numel(), _Buffers()
+    args = [b(seg_id, "seg_id", _I32, T), b(mask, "mask", _BYTE, T), T, int(n_ids),
+            b(counts, "counts", _I32, 2 * int(n_ids)), float(eps), b(loss_in, "loss_in", _F32, T),
+            b(w_out, "w_out", _F32, T), b(loss_out, "loss_out", _F32, 1), b(workspace, "workspace"),
+            _nbytes(workspace)]
+    _check(_call("opd_seq_mean_token_mean_from_counts", b, args, stream), "opd_seq_mean_token_mean_from_counts")
 
 
 def opd_kl_get_status(workspace, stream=None) -> int:

@@ -1,0 +1,61 @@
+"""One rank of the token-sharded data-parallel CPU test (torch.distributed.run, gloo).
+
+The rank takes its contiguous rows of one small packed batch (row_shards), builds its
+histogram of response ids (standing in for the device pass opd_seq_mean_token_mean_counts),
+sums it over the ranks with the library's Reducer, computes its rows' KL, dH_s and dW_s part
+with the float64 oracle under the whole batch's seq-mean-token-mean weights, and sums dW_s
+(in several buckets) and its part of the loss over the ranks. The parent test compares the
+result with one oracle call over the whole batch."""
+
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+import torch.distributed as dist  # noqa: E402
+
+import oracle  # noqa: E402
+from paper_2609_36608_gb300 import data_parallel as dp  # noqa: E402
+from paper_2609_36608_gb300 import synth  # noqa: E402
+
+
+def batch():
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="dp_small", T=300, d_s=32, d_t=48, V=200, tau=0.8,
+                     n_traj=3, traj_len=100, seed=5)
+    return w, synth.layout(w)
+
+
+def main():
+    dist.init_process_group("gloo")
+    world, rank = dist.get_world_size(), dist.get_rank()
+    w, lay = batch()
+    x = synth.hidden_and_heads(w, "cpu")
+    host = [synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")]
+    n_ids = int(lay.seg_id.max()) + 1
+    lo, hi = dp.row_shards(w.T, world, lay.mask)[rank]
+    counts = torch.zeros(2 * n_ids, dtype=torch.int32)
+    for i in range(lo, hi):
+        b = int(lay.seg_id[i])
+        if b >= 0:
+            counts[b] += int(lay.mask[i] != 0)
+            counts[n_ids + b] += 1
+    red = dp.Reducer(bucket_bytes=7 * w.d_s * 8)  # 7 vocabulary rows per bucket: 29 buckets
+    red.sum_(counts)
+    g = oracle.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+    rows = np.arange(lo, hi)
+    res = oracle.opd_kl(*host, lay.mask, g, w.tau, rows=rows, want_dH=True, want_dW=True, n_threads=1)
+    dW = torch.from_numpy(np.ascontiguousarray(res.dW_s))
+    for work in red.sum_rows_(dW, async_op=True):
+        work.wait()
+    loss = torch.tensor([float(np.sum(g[rows] * res.kl))], dtype=torch.float64)
+    red.sum_(loss)
+    np.savez(os.path.join(os.environ["OPD_TEST_OUT"], f"rank{rank}.npz"), lo=lo, hi=hi, counts=counts.numpy(),
+             kl=res.kl, dH=res.dH_s, dW=dW.numpy(), loss=loss.numpy(), buckets=len(red.buckets(w.V, w.d_s * 8)))
+    dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

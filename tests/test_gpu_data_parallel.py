@@ -1,0 +1,134 @@
+"""GPU side of token-sharded data parallelism, on one GPU: the rows of one batch are cut into
+shards as row_shards cuts them across ranks, and each shard runs through the C ABI as its
+rank would. The histogram sum that the all-reduce performs between ranks is done here by
+adding the shards' count buffers; nothing waits on another shard's kernels.
+
+Checked against the float64 oracle on the whole batch: the seq-mean-token-mean weights from
+summed counts (Appendix B.4, Eq. opd-surrogate), the per-token KL, dH_s rows, dW_s summed
+over the shards, and the batch loss."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36608_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+KL_ABS, KL_REL, GRAD_REL = 1e-4, 2e-3, 1e-2
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2609_36608_gb300 import build
+    build.build()
+    from paper_2609_36608_gb300 import opd_kl
+    return opd_kl
+
+
+def _rel(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def _batch(**kw):
+    base = dict(name="dp", T=900, d_s=192, d_t=256, V=1500, tau=0.8, n_traj=3, traj_len=300, seed=61)
+    base.update(kw)
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], **base)
+    return w, synth.layout(w)
+
+
+@pytest.mark.parametrize("world", [1, 2, 3])
+def test_weights_from_counts_summed_over_shards(lib, oracle_mod, world):
+    from paper_2609_36608_gb300 import data_parallel as dp
+    for w, lay in (_batch(), _batch(name="dp_ragged", T=4000, n_traj=8, traj_len=500, seed=62)):
+        n_ids = int(lay.seg_id.max()) + 1
+        seg = torch.from_numpy(lay.seg_id).cuda()
+        mask = torch.from_numpy(lay.mask).cuda()
+        shards = dp.row_shards(w.T, world, lay.mask)
+        ws = [torch.empty(lib.opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8, device="cuda")
+              for _ in shards]
+        counts = [torch.full((2 * n_ids,), -7, dtype=torch.int32, device="cuda") for _ in shards]
+        for (lo, hi), c, s in zip(shards, counts, ws):
+            lib.opd_seq_mean_token_mean_counts(seg[lo:hi], mask[lo:hi], n_ids, c, s)
+        total = sum(counts)  # what the all-reduce leaves on every rank
+        sup = np.bincount(lay.seg_id[(lay.seg_id >= 0) & (lay.mask != 0)], minlength=n_ids)
+        rows = np.bincount(lay.seg_id[lay.seg_id >= 0], minlength=n_ids)
+        np.testing.assert_array_equal(total.cpu().numpy(), np.concatenate([sup, rows]))
+        loss_in = torch.from_numpy(np.random.default_rng(world).random(w.T).astype(np.float32)).cuda()
+        wt = torch.full((w.T,), float("nan"), device="cuda")
+        parts = torch.zeros(len(shards), device="cuda")
+        for k, ((lo, hi), s) in enumerate(zip(shards, ws)):
+            lib.opd_seq_mean_token_mean_from_counts(seg[lo:hi], mask[lo:hi], n_ids, total, 1e-8, loss_in[lo:hi],
+                                                    wt[lo:hi], parts[k:k + 1], s)
+        torch.cuda.synchronize()
+        for s in ws:
+            assert lib.opd_kl_get_status(s) == lib.OPD_OK
+        ref = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+        np.testing.assert_allclose(wt.cpu().numpy(), ref, rtol=2e-7, atol=0)
+        want = float(np.sum(ref * loss_in.cpu().numpy().astype(np.float64)))
+        assert abs(float(parts.sum()) - want) <= 1e-6 * abs(want)
+
+
+def test_counts_report_an_id_beyond_n_ids(lib):
+    seg = torch.tensor([0, 1, 5, -1], dtype=torch.int32, device="cuda")
+    mask = torch.ones(4, dtype=torch.uint8, device="cuda")
+    ws = torch.empty(lib.opd_seq_mean_token_mean_workspace_size(2), dtype=torch.uint8, device="cuda")
+    c = torch.empty(4, dtype=torch.int32, device="cuda")
+    lib.opd_seq_mean_token_mean_counts(seg, mask, 2, c, ws)
+    w = torch.empty(4, device="cuda")
+    lib.opd_seq_mean_token_mean_from_counts(seg, mask, 2, c, 1e-8, None, w, None, ws)
+    assert lib.opd_kl_get_status(ws) == lib.OPD_ERR_INVALID_ARG  # the histogram pass's report survives
+    assert c.cpu().tolist() == [1, 1, 1, 1]
+    assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+
+
+@pytest.mark.parametrize("world", [1, 2, 3])
+def test_sharded_step_equals_the_whole_batch(lib, oracle_mod, world):
+    """Each shard runs ShardedSeqMeanKL's calls (counts, summed counts, weights, fused step,
+    its part of the loss); the shards' dW_s parts and losses are then summed as the all-reduce
+    would sum them. With one shard this is ShardedSeqMeanKL.step itself."""
+    from paper_2609_36608_gb300 import data_parallel as dp
+    w, lay = _batch()
+    x = synth.hidden_and_heads(w, "cuda")
+    n_ids = int(lay.seg_id.max()) + 1
+    seg = torch.from_numpy(lay.seg_id).cuda()
+    mask = torch.from_numpy(lay.mask).cuda()
+    shards = dp.row_shards(w.T, world, lay.mask)
+    steps = [dp.ShardedSeqMeanKL(hi - lo, w.d_s, w.d_t, w.V, n_ids, w.tau) for lo, hi in shards]
+    dH = torch.full((w.T, w.d_s), float("nan"), device="cuda")
+    dWs = [torch.full((w.V, w.d_s), float("nan"), device="cuda") for _ in shards]
+    if world == 1:
+        steps[0].step(x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, seg, dH, dWs[0])
+        kl, loss, dW = steps[0].kl, steps[0].loss, dWs[0]
+    else:
+        counts = []
+        for st, (lo, hi) in zip(steps, shards):
+            lib.opd_seq_mean_token_mean_counts(seg[lo:hi], mask[lo:hi], n_ids, st.counts, st.seq_ws)
+            counts.append(st.counts)
+        total = sum(counts)
+        kl = torch.empty(w.T, device="cuda")
+        loss = torch.zeros(1, device="cuda")
+        for st, (lo, hi), dW_k in zip(steps, shards, dWs):
+            st.counts.copy_(total)
+            args = (seg[lo:hi], mask[lo:hi], n_ids, st.counts, st.eps)
+            lib.opd_seq_mean_token_mean_from_counts(*args, None, st.weights, None, st.seq_ws)
+            lib.opd_kl_fwd_bwd(st.problem, x["H_s"][lo:hi], x["H_t"][lo:hi], x["W_s"], x["W_t"], mask[lo:hi],
+                               st.weights, st.kl, st.stats, dH[lo:hi], dW_k, False, st.ws)
+            lib.opd_seq_mean_token_mean_from_counts(*args, st.kl, None, st.loss, st.seq_ws)
+            kl[lo:hi] = st.kl
+            loss += st.loss
+        dW = sum(dWs)
+    torch.cuda.synchronize()
+    for st in steps:
+        assert lib.opd_kl_get_status(st.ws) == lib.OPD_OK and lib.opd_kl_get_status(st.seq_ws) == lib.OPD_OK
+    host = [synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")]
+    g = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+    ref = oracle_mod.opd_kl(*host, lay.mask, g.astype(np.float32).astype(np.float64), w.tau)
+    got = kl.cpu().numpy().astype(np.float64)
+    assert (np.abs(got - ref.kl) <= KL_ABS + KL_REL * np.abs(ref.kl)).all()
+    assert _rel(dH.cpu().numpy(), ref.dH_s) <= GRAD_REL
+    assert _rel(dW.cpu().numpy(), ref.dW_s) <= GRAD_REL
+    want = float(np.sum(g * ref.kl))
+    assert abs(float(loss[0]) - want) <= 1e-4 * abs(want) + 1e-7
