@@ -184,6 +184,19 @@ def sum_over_ranks(x: int, world: int, device) -> int:
     return int(t.item())
 
 
+def workload_from_args(args):
+    """The named workload; --trajectories N shrinks a packed workload to N trajectories of its
+    length (the same shapes per row and the same layout generator: the small case of the same
+    kernels that the ncu captures use)."""
+    w = synth.WORKLOADS[args.workload]
+    n = getattr(args, "trajectories", 0) or 0
+    if n:
+        if w.layout != "packed":
+            raise SystemExit("--trajectories applies to the packed workloads only")
+        w = synth.scaled(w, name=f"{w.name}_{n}traj", n_traj=n, T=n * w.traj_len)
+    return w
+
+
 def rank_workload(w, rank: int):
     """Each rank's own batch under data parallelism: rank 0 keeps the workload's seed (its
     batch is the single-GPU batch), rank k draws another packed batch of the same shape."""
@@ -258,7 +271,7 @@ def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
         return 0
-    w = synth.WORKLOADS[args.workload]
+    w = workload_from_args(args)
     lay = synth.layout(w)
     gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
     x = synth.hidden_and_heads(w, gen_dev)
@@ -515,7 +528,7 @@ def run_gpu(args):
     build.build()
     from paper_2609_36608_gb300 import opd_kl
 
-    w = rank_workload(synth.WORKLOADS[args.workload], rank)
+    w = rank_workload(workload_from_args(args), rank)
     lay = synth.layout(w)
     R = int(lay.mask.sum())
     R_job = sum_over_ranks(R, world, dev)  # supervised rows of all ranks' batches per step
@@ -715,7 +728,7 @@ def run_calibration(args):
     b = torch.randn(8192, 8192, device="cuda", dtype=torch.bfloat16)
     sustained("cublas_bf16_8192", lambda: torch.matmul(a, b), 2.0 * 8192 ** 3)
     del a, b
-    w = synth.WORKLOADS[args.workload]
+    w = workload_from_args(args)
     lay = synth.layout(w)
     R = int(lay.mask.sum())
     x = synth.hidden_and_heads(w, "cuda")
@@ -744,6 +757,8 @@ def main():
                     help="kl: the reverse-KL step (default, the headline); kl_seqmean: the same step "
                          "with the paper's batch loss aggregated on the device; surrogate: the "
                          "sampled-token dual-clip surrogate; score: teacher token scoring")
+    ap.add_argument("--trajectories", type=int, default=0, metavar="N",
+                    help="a packed workload cut to N trajectories (a small case for profiling)")
     ap.add_argument("--cpu-rows", type=int, default=48, help="row sample of the CPU-oracle baseline")
     ap.add_argument("--cpu-rows-1t", type=int, default=4, help="rows of the one-core CPU-oracle sample")
     ap.add_argument("--ref-rows", type=int, default=16, help="rows per step of --impl reference (the oracle splits rows over the host cores)")
