@@ -119,16 +119,21 @@ class ClockSampler:
                 self.proc.kill()
             self.thread.join(timeout=5)
 
-    def summary(self):
-        if not self.rows:
+    def mark(self) -> int:
+        return len(self.rows)
+
+    def summary(self, start: int = 0, end=None):
+        """Median SM clock, maximum, throttle reasons and peak power of the samples [start, end)."""
+        rows = self.rows[start:end]
+        if not rows:
             return None
-        sm = [float(r[0]) for r in self.rows if re.match(r"^[\d.]+$", r[0])]
-        mx = [float(r[1]) for r in self.rows if re.match(r"^[\d.]+$", r[1])]
+        sm = [float(r[0]) for r in rows if re.match(r"^[\d.]+$", r[0])]
+        mx = [float(r[1]) for r in rows if re.match(r"^[\d.]+$", r[1])]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[4 + i].lower().startswith("active")})
-        pw = [float(r[2]) for r in self.rows if re.match(r"^[\d.]+$", r[2])]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower().startswith("active")})
+        pw = [float(r[2]) for r in rows if re.match(r"^[\d.]+$", r[2])]
         return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(self.rows), "power_w_max": max(pw) if pw else None}
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
 
 
 def choose_peak(clocks, peaks, peak_src):
@@ -543,10 +548,35 @@ def run_gpu(args):
     torch.cuda.synchronize()
     if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
         raise RuntimeError("device status after warm-up is not OK")
-    if sampler:
-        sampler.rows.clear()  # keep only samples taken while the timed steps run
+    # Per-kernel times for the roofline come from K more steps with every library launch
+    # bracketed by CUDA events on the launch stream: half of them just before the timed
+    # region and half just after it, so that under the power limiter their clocks average out
+    # to the timed region's. The timed region itself runs with the per-launch events off.
+    prof = {}
+    prof_ms = [0.0]
+    prof_marks = []
+
+    def kernel_pass(n):
+        if n <= 0:
+            return
+        opd_kl.opd_kl_profile_start()
+        q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        i0 = sampler.mark() if sampler else 0
+        q0.record()
+        for _ in range(n):
+            step(inputs)
+        q1.record()
+        torch.cuda.synchronize()
+        prof_marks.append((i0, sampler.mark() if sampler else 0))
+        for name, (cnt, tot) in opd_kl.opd_kl_profile_stop().items():
+            c0, t0 = prof.get(name, (0, 0.0))
+            prof[name] = (c0 + cnt, t0 + tot)
+        prof_ms[0] += q0.elapsed_time(q1)
+
+    kernel_pass(args.steps // 2)
     barrier(world)
     torch.cuda.synchronize()
+    mark0 = sampler.mark() if sampler else 0
     # the timed region: K steps, no per-launch events (the library's kernel timing is off)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]  # end of each step
@@ -563,21 +593,18 @@ def run_gpu(args):
     ms = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_step = ms / args.steps
     value = whole_job_rate(R_job, args.steps, 1, ms)
-    clocks = sampler.summary() if sampler else None  # samples of the timed region only
+    clocks = sampler.summary(mark0, sampler.mark()) if sampler else None  # the timed region's samples
 
-    # per-kernel times for the roofline: a second pass of the same K steps with every
-    # library launch bracketed by CUDA events on the launch stream
-    opd_kl.opd_kl_profile_start()
-    p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    p0.record()
-    for k in range(args.steps):
-        step(inputs)
-    p1.record()
-    torch.cuda.synchronize()
-    prof = opd_kl.opd_kl_profile_stop()
-    ms_profiled = p0.elapsed_time(p1) / args.steps
+    kernel_pass(args.steps - args.steps // 2)
+    ms_profiled = prof_ms[0] / args.steps
     if sampler:
         sampler.stop()
+    clocks_kernel_pass = None
+    if sampler and prof_marks:
+        rows = [r for a, b in prof_marks for r in sampler.rows[a:b]]
+        saved, sampler.rows = sampler.rows, rows
+        clocks_kernel_pass = sampler.summary()
+        sampler.rows = saved
     if opd_kl.opd_kl_get_status(ws) != opd_kl.OPD_OK:
         raise RuntimeError("device status after the per-kernel pass is not OK")
 
@@ -662,7 +689,7 @@ def run_gpu(args):
         "metric": PATH_METRICS[args.path], "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step,
         "ms_per_step_median": float(np.median(per_step)), "ms_per_step_min_max": [min(per_step), max(per_step)],
-        "ms_per_step_kernel_pass": ms_profiled,
+        "ms_per_step_kernel_pass": ms_profiled, "clocks_kernel_pass": clocks_kernel_pass,
         "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded counter-based generator, packed multi-turn layout with masked observations "
