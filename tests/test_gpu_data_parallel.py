@@ -132,3 +132,45 @@ def test_sharded_step_equals_the_whole_batch(lib, oracle_mod, world):
     assert _rel(dW.cpu().numpy(), ref.dW_s) <= GRAD_REL
     want = float(np.sum(g * ref.kl))
     assert abs(float(loss[0]) - want) <= 1e-4 * abs(want) + 1e-7
+
+
+def test_bench_data_parallel_step_in_a_process_group_of_one(lib, oracle_mod, tmp_path):
+    """bench.py's N > 1 step (path_setup with world > 1: global response ids, ShardedSeqMeanKL,
+    the collectives) run as rank 0 of a one-rank NCCL process group: the collectives are then
+    identities, and the loss and gradients must equal one whole-batch opd_kl_seq_mean_fwd_bwd call."""
+    import torch.distributed as dist
+    import bench
+    from paper_2609_36608_gb300 import data_parallel as dp
+    w, lay = _batch(name="dp_bench", T=1200, n_traj=4, seed=63)
+    x = synth.hidden_and_heads(w, "cuda")
+    dev = torch.device("cuda", torch.cuda.current_device())
+    dist.init_process_group("nccl", init_method=f"file://{tmp_path}/pg", world_size=1, rank=0)
+    try:
+        inputs, step, result, ws, executed, algorithmic = bench.path_setup("kl", w, lay, x, dev, lib, world=2,
+                                                                           rank=0)
+        step(inputs)
+        torch.cuda.synchronize()
+        assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+        assert not dp.Reducer().active  # one rank: the sums over ranks leave every buffer as it is
+        loss = float(result[0])
+        kl = step.outputs["kl"].cpu().numpy()
+        dH = step.outputs["dH"].cpu().numpy()
+    finally:
+        dist.destroy_process_group()
+    n_ids = int(lay.seg_id.max()) + 1
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    ws2 = lib.allocate_seq_mean_workspace(prob, n_ids)
+    loss2, kl2, st2 = torch.empty(1, device="cuda"), torch.empty(w.T, device="cuda"), torch.empty(w.T, 3, device="cuda")
+    dH2, dW2 = torch.empty(w.T, w.d_s, device="cuda"), torch.empty(w.V, w.d_s, device="cuda")
+    lib.opd_kl_seq_mean_fwd_bwd(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], torch.from_numpy(lay.mask).cuda(),
+                                torch.from_numpy(lay.seg_id).cuda(), n_ids, 1e-8, loss2, kl2, st2, dH2, dW2, False,
+                                ws2)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(kl, kl2.cpu().numpy())
+    assert _rel(dH, dH2.cpu().numpy().astype(np.float64)) < 1e-5
+    assert abs(loss - float(loss2[0])) <= 1e-6 * abs(float(loss2[0]))
+    g = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+    ref = oracle_mod.opd_kl(*(synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")), lay.mask,
+                            g.astype(np.float32).astype(np.float64), w.tau, want_dW=False)
+    want = float(np.sum(g * ref.kl))
+    assert abs(loss - want) <= 1e-4 * abs(want) + 1e-7
