@@ -237,9 +237,10 @@ opd_status opd_seq_mean_token_mean_weights(const int32_t* seg_id, const uint8_t*
  * seg_id [T] int32 and mask [T] uint8 in device memory, response ids in [0, n_ids) (ids < 0
  * mark rows outside every response; an id >= n_ids sets the workspace status, reported as
  * OPD_ERR_INVALID_ARG by opd_kl_get_status). Writes w_out [T] (device, may be NULL) and,
- * when loss_in [T] and loss_out [1] are both given, loss_out[0] = sum_i w_i loss_in[i],
- * which is the paper's L for per-token losses loss_in (accumulated in double; the
- * summation order is not fixed). At least one of the two outputs must be requested.
+ * when loss_out [1] is given, loss_out[0] = sum_i w_i loss_in[i], which is the paper's L for
+ * per-token losses loss_in [T] (accumulated in double; the summation order is not fixed).
+ * loss_in is required with loss_out unless T = 0 (then L = 0). At least one of the two
+ * outputs must be requested.
  * The workspace (device, 256-byte aligned) holds opd_seq_mean_token_mean_workspace_size(n_ids)
  * bytes; it starts with the status word opd_kl_get_status reads. */
 size_t opd_seq_mean_token_mean_workspace_size(int64_t n_ids);
@@ -258,9 +259,10 @@ opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* 
  *      sets the workspace status (OPD_ERR_INVALID_ARG from opd_kl_get_status).
  *   2. The caller sums counts over the processes (an all-reduce of 2 n_ids int32 values).
  *   3. opd_seq_mean_token_mean_from_counts takes the summed counts and writes this process's
- *      weights w_out [T] (may be NULL) and, when loss_in [T] and loss_out [1] are given,
- *      loss_out[0] = sum over this process's rows of w_i loss_in[i] (in double, in no fixed
- *      order). The sum of loss_out over the processes is the batch loss L.
+ *      weights w_out [T] (may be NULL) and, when loss_out [1] is given, loss_out[0] = sum over
+ *      this process's rows of w_i loss_in[i] (in double, in no fixed order; loss_in [T] is
+ *      required unless T = 0, where the part is 0). The sum of loss_out over the processes is
+ *      the batch loss L. At least one of w_out and loss_out must be given.
  * Response ids are global ids in [0, n_ids) (ids < 0 mark rows outside every response).
  * With one process the result equals opd_seq_mean_token_mean_device. Workspaces as for
  * opd_seq_mean_token_mean_device (the status word of step 1 stays set through step 3).

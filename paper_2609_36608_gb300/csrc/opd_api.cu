@@ -688,22 +688,23 @@ opd_status opd_seq_mean_token_mean_device(const int32_t* seg_id, const uint8_t* 
   if (T < 0 || T > (int64_t)0x7FFF0000 || n_ids < 1 || n_ids > (int64_t)0x7FFF0000 || !(eps >= 0.0f))
     return OPD_ERR_INVALID_ARG;
   if (T > 0 && (!seg_id || !mask)) return OPD_ERR_INVALID_ARG;
-  if (!w_out && !(loss_in && loss_out)) return OPD_ERR_INVALID_ARG;
+  // the loss is requested by loss_out; its input may be absent only when there are no rows
+  if ((loss_out && T > 0 && !loss_in) || (!w_out && !loss_out)) return OPD_ERR_INVALID_ARG;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < opd_seq_mean_token_mean_workspace_size(n_ids))
     return OPD_ERR_INVALID_ARG;
   const DeviceInfo dev = device_info();
   if (dev.sm_count <= 0) return OPD_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   OPD_CUDA(timed("seq_mean_token_mean", s, [&] {
-    return launch_seq_mean_token_mean(seg_id, mask, (int32_t)T, (int32_t)n_ids, eps, loss_in, w_out,
-                                      loss_in ? loss_out : nullptr, static_cast<Ctrl*>(workspace), true,
+    return launch_seq_mean_token_mean(seg_id, mask, (int32_t)T, (int32_t)n_ids, eps, loss_out ? loss_in : nullptr,
+                                      w_out, loss_out, static_cast<Ctrl*>(workspace), true,
                                       static_cast<uint8_t*>(workspace) + sizeof(Ctrl), dev.sm_count, s);
   }));
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
   if (env_flag("OPD_KL_SYNC_CHECK")) {
     Ctrl* ctrl = static_cast<Ctrl*>(workspace);
     OPD_CUDA(launch_check_finite(w_out, w_out ? (size_t)T : 0, ctrl, dev.sm_count, s));
-    OPD_CUDA(launch_check_finite(loss_in ? loss_out : nullptr, 1, ctrl, dev.sm_count, s));
+    OPD_CUDA(launch_check_finite(loss_out, 1, ctrl, dev.sm_count, s));
     return opd_kl_get_status(workspace, workspace_bytes, stream);
   }
   return OPD_OK;
@@ -734,7 +735,8 @@ opd_status opd_seq_mean_token_mean_from_counts(const int32_t* seg_id, const uint
   if (T < 0 || T > (int64_t)0x7FFF0000 || n_ids < 1 || n_ids > (int64_t)0x3FFF0000 || !(eps >= 0.0f))
     return OPD_ERR_INVALID_ARG;
   if ((T > 0 && (!seg_id || !mask)) || !counts) return OPD_ERR_INVALID_ARG;
-  if (!w_out && !(loss_in && loss_out)) return OPD_ERR_INVALID_ARG;
+  // the loss is requested by loss_out; its input may be absent only when there are no rows
+  if ((loss_out && T > 0 && !loss_in) || (!w_out && !loss_out)) return OPD_ERR_INVALID_ARG;
   if (!workspace || !aligned(workspace, 256) || workspace_bytes < opd_seq_mean_token_mean_workspace_size(n_ids))
     return OPD_ERR_INVALID_ARG;
   const DeviceInfo dev = device_info();
@@ -742,14 +744,14 @@ opd_status opd_seq_mean_token_mean_from_counts(const int32_t* seg_id, const uint
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Ctrl* ctrl = static_cast<Ctrl*>(workspace);
   OPD_CUDA(timed("seq_from_counts", s, [&] {
-    return launch_seq_from_counts(seg_id, mask, (int32_t)T, (int32_t)n_ids, counts, eps, loss_in, w_out,
-                                  loss_in ? loss_out : nullptr, ctrl, static_cast<uint8_t*>(workspace) + sizeof(Ctrl),
+    return launch_seq_from_counts(seg_id, mask, (int32_t)T, (int32_t)n_ids, counts, eps, loss_out ? loss_in : nullptr,
+                                  w_out, loss_out, ctrl, static_cast<uint8_t*>(workspace) + sizeof(Ctrl),
                                   dev.sm_count, s);
   }));
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
   if (env_flag("OPD_KL_SYNC_CHECK")) {
     OPD_CUDA(launch_check_finite(w_out, w_out ? (size_t)T : 0, ctrl, dev.sm_count, s));
-    OPD_CUDA(launch_check_finite(loss_in ? loss_out : nullptr, 1, ctrl, dev.sm_count, s));
+    OPD_CUDA(launch_check_finite(loss_out, 1, ctrl, dev.sm_count, s));
     return opd_kl_get_status(workspace, workspace_bytes, stream);
   }
   return OPD_OK;

@@ -138,6 +138,28 @@ def test_seq_mean_token_mean_device_arguments(lib):
     assert rc == lib.OPD_ERR_INVALID_ARG
 
 
+def test_seq_mean_counts_arguments(lib):
+    vp = ctypes.c_void_p
+    fake = vp(1 << 20)
+    n = ctypes.c_size_t(lib.opd_seq_mean_token_mean_workspace_size(8))
+    counts = lambda T, n_ids, c: lib.call_raw("opd_seq_mean_token_mean_counts", fake, fake, ctypes.c_int64(T),
+                                              ctypes.c_int64(n_ids), c, fake, n, None)
+    assert counts(4, 0, fake) == lib.OPD_ERR_INVALID_ARG
+    assert counts(4, 8, None) == lib.OPD_ERR_INVALID_ARG
+    assert counts(-1, 8, fake) == lib.OPD_ERR_INVALID_ARG
+    assert lib.call_raw("opd_seq_mean_token_mean_counts", fake, fake, ctypes.c_int64(4), ctypes.c_int64(8), fake,
+                        fake, ctypes.c_size_t(64), None) == lib.OPD_ERR_INVALID_ARG  # workspace too small
+
+    def from_counts(T, loss_in, w_out, loss_out, eps=1e-8):
+        return lib.call_raw("opd_seq_mean_token_mean_from_counts", fake, fake, ctypes.c_int64(T), ctypes.c_int64(8),
+                            fake, ctypes.c_float(eps), loss_in, w_out, loss_out, fake, n, None)
+    assert from_counts(4, None, None, None) == lib.OPD_ERR_INVALID_ARG  # nothing requested
+    assert from_counts(4, None, None, fake) == lib.OPD_ERR_INVALID_ARG  # a loss of rows without their losses
+    assert from_counts(4, fake, fake, None, eps=-1.0) == lib.OPD_ERR_INVALID_ARG
+    # no rows: the loss needs no input (the call then stops at the missing GPU, or runs)
+    assert from_counts(0, None, None, fake) != lib.OPD_ERR_INVALID_ARG
+
+
 def test_kl_seq_mean_arguments(lib):
     p = lib.make_problem(1000, 64, 64, 500, lib.OPD_DTYPE_BF16, 1.0)
     base = lib.opd_kl_workspace_size(p)

@@ -174,3 +174,40 @@ def test_bench_data_parallel_step_in_a_process_group_of_one(lib, oracle_mod, tmp
                             g.astype(np.float32).astype(np.float64), w.tau, want_dW=False)
     want = float(np.sum(g * ref.kl))
     assert abs(loss - want) <= 1e-4 * abs(want) + 1e-7
+
+
+def test_shards_with_no_rows_and_loss_only_requests(lib, oracle_mod):
+    """Degenerate shards: a rank whose row range is empty (T = 0) contributes a zero histogram and
+    nothing else; a rank whose rows are all masked contributes only its responses' presence.
+    from_counts with the loss alone (no weights buffer) gives that rank's part of L."""
+    from paper_2609_36608_gb300 import data_parallel as dp
+    w, lay = _batch(name="dp_edge", T=600, n_traj=2, seed=64)
+    n_ids = int(lay.seg_id.max()) + 1
+    seg = torch.from_numpy(lay.seg_id).cuda()
+    mask = torch.from_numpy(lay.mask).cuda()
+    # rank 0: nothing; rank 1: the first half with its mask cleared; rank 2: the rest
+    half = w.T // 2
+    shards = [(0, 0), (0, half), (half, w.T)]
+    masks = [mask[0:0], torch.zeros(half, dtype=torch.uint8, device="cuda"), mask[half:]]
+    eff_mask = np.concatenate([np.zeros(half, np.uint8), lay.mask[half:]])
+    ws = [torch.empty(lib.opd_seq_mean_token_mean_workspace_size(n_ids), dtype=torch.uint8, device="cuda")
+          for _ in shards]
+    counts = [torch.full((2 * n_ids,), 5, dtype=torch.int32, device="cuda") for _ in shards]
+    for (lo, hi), m, c, s in zip(shards, masks, counts, ws):
+        lib.opd_seq_mean_token_mean_counts(seg[lo:hi], m, n_ids, c, s)
+    assert (counts[0] == 0).all()
+    total = sum(counts)
+    loss_in = torch.from_numpy(np.random.default_rng(3).random(w.T).astype(np.float32)).cuda()
+    parts = torch.full((3,), float("nan"), device="cuda")
+    for k, ((lo, hi), m, s) in enumerate(zip(shards, masks, ws)):
+        lib.opd_seq_mean_token_mean_from_counts(seg[lo:hi], m, n_ids, total, 1e-8, loss_in[lo:hi], None,
+                                                parts[k:k + 1], s)
+    torch.cuda.synchronize()
+    for s in ws:
+        assert lib.opd_kl_get_status(s) == lib.OPD_OK
+    ref = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, eff_mask)
+    p = parts.cpu().numpy().astype(np.float64)
+    assert p[0] == 0.0 and p[1] == 0.0
+    want = float(np.sum(ref * loss_in.cpu().numpy().astype(np.float64)))
+    assert abs(p.sum() - want) <= 1e-6 * abs(want)
+    assert dp.row_shards(w.T, 3, np.zeros(w.T, np.uint8)) == [(0, 0), (0, 0), (0, w.T)]

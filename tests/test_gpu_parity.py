@@ -91,6 +91,23 @@ def _full_check(lib, oracle_mod, w, mask=None, g=None, tight=False, **kw):
     return out, ref, x
 
 
+def test_forward_only_workspace_with_every_row_masked(lib):
+    """R = 0 with the forward-only workspace, on both element types: zeros out, status OK."""
+    for dtype, tdt in ((lib.OPD_DTYPE_BF16, torch.bfloat16), (lib.OPD_DTYPE_F32, torch.float32)):
+        T, ds, dt, V = 300, 64, 96, 500
+        prob = lib.make_problem(T, ds, dt, V, dtype, 1.0)
+        ws = torch.empty(lib.opd_kl_forward_workspace_size(prob), dtype=torch.uint8, device="cuda")
+        H_s, H_t = torch.ones(T, ds, dtype=tdt, device="cuda"), torch.ones(T, dt, dtype=tdt, device="cuda")
+        W_s, W_t = torch.ones(V, ds, dtype=tdt, device="cuda"), torch.ones(V, dt, dtype=tdt, device="cuda")
+        mask = torch.zeros(T, dtype=torch.uint8, device="cuda")
+        kl = torch.full((T,), float("nan"), device="cuda")
+        stats = torch.full((T, 3), float("nan"), device="cuda")
+        lib.opd_kl_forward(prob, H_s, H_t, W_s, W_t, mask, kl, stats, ws)
+        torch.cuda.synchronize()
+        assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+        assert (kl == 0).all() and (stats == 0).all()
+
+
 @pytest.mark.parametrize("which", ["tiny_fp32", "bf16"])
 def test_forward_and_scoring_with_the_forward_only_workspace(lib, oracle_mod, which):
     """opd_kl_forward and opd_score_tokens given exactly opd_kl_forward_workspace_size bytes (no dz
