@@ -110,8 +110,10 @@ class ShardedSeqMeanKL:
     rows of a batch sharded by rows (see the module docstring for the steps).
 
     Construct once per shape on each rank; `step` then runs without host synchronisation.
+    T is this rank's row count (its shard of the batch); d_s, d_t and V are the heads' sizes.
     `n_ids` is the number of global response ids of the whole batch (every rank passes the
-    same value); seg_id holds global ids."""
+    same value); seg_id holds global ids. The workspaces are allocated here, once, through
+    PyTorch; the library itself allocates nothing."""
 
     def __init__(self, T: int, d_s: int, d_t: int, V: int, n_ids: int, temperature: float = 1.0,
                  eps: float = 1e-8, device="cuda", group=None, bucket_bytes: int = 256 << 20,
