@@ -59,13 +59,20 @@ def log(*a):
 
 
 def load_peaks():
+    """The measured peaks (or the fallback) and, when recorded, the median SM clock of the
+    sustained bf16 measurement (key "sustained_mhz")."""
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(path) as f:
             d = json.load(f)
-        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+        out = {k: float(d[k]) for k in FALLBACK_PEAKS}
     except (OSError, KeyError, ValueError):
         return dict(FALLBACK_PEAKS), "fallback"
+    try:
+        out["sustained_mhz"] = float(d["clocks_under_load"]["sm_mhz_median"])
+    except (KeyError, TypeError, ValueError):
+        pass
+    return out, "measured"
 
 
 # --------------------------------------------------------------------- clocks
@@ -138,12 +145,15 @@ class ClockSampler:
 
 def choose_peak(clocks, peaks, peak_src):
     """The bf16 denominator for a kernel timed inside the benchmark's step: the sustained
-    figure when the step ran under the power limiter (sw_power_cap seen, or the median SM
-    clock below 95% of its maximum), else the burst figure. Without a clock record the
-    burst figure (the larger one) is used. Returns (peak, description)."""
+    figure when the kernel ran under the power limiter (sw_power_cap seen, or the median SM
+    clock below 95% of its maximum) at a clock no more than 5% above the one the sustained
+    figure was measured at; else the burst figure. Without a clock record the burst figure
+    (the larger one) is used. Returns (peak, description)."""
     capped = bool(clocks) and (
         "sw_power_cap" in (clocks.get("reasons") or [])
         or (clocks.get("sm_mhz") and clocks.get("sm_max_mhz") and clocks["sm_mhz"] < 0.95 * clocks["sm_max_mhz"]))
+    if capped and clocks.get("sm_mhz") and peaks.get("sustained_mhz"):
+        capped = clocks["sm_mhz"] <= 1.05 * peaks["sustained_mhz"]
     if capped:
         return peaks["bf16_tflops_sustained"], f"bf16_tflops_sustained of {peak_src} (the step ran power-capped)"
     return peaks["bf16_tflops"], f"bf16_tflops (burst) of {peak_src} (the step ran at full clock)"
@@ -673,12 +683,15 @@ def run_gpu(args):
     if dom:
         per_launch = path_kernel_flops(args.path, dom, w, R)
         achieved = per_launch / (kernels[dom]["ms_per_launch"] / 1000.0) / 1e12
-        peak, peak_desc = choose_peak(clocks, peaks, peak_src)
+        # the per-kernel times come from the kernel passes, so their clocks pick the peak
+        peak, peak_desc = choose_peak(clocks_kernel_pass or clocks, peaks, peak_src)
         traffic = recorded_traffic(dom, w.name, args.path)
         roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak, "traffic": traffic, "peak_source": peak_desc,
                     "frac_of_burst": achieved / peaks["bf16_tflops"],
                     "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
+                    # the same kernel at its kernel-pass share of the timed region's step time
+                    "frac_at_timed_step": achieved / peak * ms_profiled / ms_step,
                     "algorithmic_flops_per_launch": per_launch}
 
     cpu, parity = None, None

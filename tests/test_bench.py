@@ -41,6 +41,14 @@ def test_peak_follows_the_clock_record():
     assert b.choose_peak(low_clock, peaks, "measured")[0] == 1749.0
     assert b.choose_peak(full, peaks, "measured")[0] == 1926.0
     assert b.choose_peak(None, peaks, "measured")[0] == 1926.0
+    # with the clock of the sustained measurement known: a capped kernel running well above
+    # that clock is held to the burst figure, one at about that clock to the sustained one
+    timed = dict(peaks, sustained_mhz=1507.0)
+    assert b.choose_peak(capped, timed, "measured")[0] == 1749.0  # 1545 <= 1.05 * 1507
+    assert b.choose_peak({"sm_mhz": 1811.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"]}, timed,
+                         "measured")[0] == 1926.0
+    p, src = b.load_peaks()
+    assert src in ("measured", "fallback") and p["bf16_tflops"] > 0
 
 
 def test_whole_job_rate_counts_every_rank_over_the_slowest_time():
