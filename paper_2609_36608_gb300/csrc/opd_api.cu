@@ -381,7 +381,7 @@ opd_status forward_body(const Call& c, const Maps& m, float* kl_out, float* stat
   OPD_CUDA(timed("fused_logits_fwd", c.s,
                  [&] { return launch_fused_forward(m.hs, m.ht, m.ws, m.wt, fp, c.dev.sm_count, c.s); }));
   OPD_CUDA(timed("combine", c.s, [&] {
-    return launch_combine(fp.partials, c.pos(), c.ctrl(), (int32_t)c.p.T, (int32_t)c.L.T_pad, kl_out, stats,
+    return launch_combine(fp.partials, c.pos(), c.idx(), c.ctrl(), (int32_t)c.p.T, (int32_t)c.L.T_pad, kl_out, stats,
                           seq ? seq->weights : nullptr, seq ? seq_mean_token_mean_acc(seq->scratch) : nullptr,
                           c.dev.sm_count, c.s);
   }));

@@ -145,52 +145,85 @@ __device__ __forceinline__ void merge_partial(float& ms, float& ss, float& as, f
   mt = Mt;
 }
 
-// One warp per token row: the lanes take the vocabulary splits' partials, then merge
-// them by shuffles. With weights, sum_i weights[i] KL_i is also added to *loss_acc.
-__global__ void k_combine(const float* __restrict__ part, const int32_t* __restrict__ pos,
-                          const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
-                          float* __restrict__ stats, const float* __restrict__ weights, double* loss_acc) {
+// Rows in blocks of 32 consecutive gathered rows, four warps per block: warp g takes the
+// vocabulary splits g, g + 4, ... of all 32 rows, so each load reads 32 consecutive floats of
+// one statistics plane (the partials are laid out [split][5][row]). The four running merges
+// meet in shared memory and warp 0 finishes the rows. idx maps a gathered row to its token
+// row (NULL: the identity, for schedules over every token row); pos[i] != r marks a row that
+// was computed but is not supervised. With weights, sum_i weights[i] KL_i is added to
+// *loss_acc. Rows outside the supervised set get zeros.
+constexpr int kCombineGroups = 4;
+__global__ void __launch_bounds__(32 * kCombineGroups)
+    k_combine(const float* __restrict__ part, const int32_t* __restrict__ pos, const int32_t* __restrict__ idx,
+              const Ctrl* __restrict__ ctrl, int32_t T, int32_t T_pad, float* __restrict__ kl_out,
+              float* __restrict__ stats, const float* __restrict__ weights, double* loss_acc) {
+  __shared__ float sh[kCombineGroups - 1][5][32];
+  const int R = ctrl->R;
   const int n_vs = ctrl->n_vsplit;
   const int h0 = ctrl->half_tile - 1;  // first row of a half-height tile, or -1
   const size_t plane = (size_t)T_pad;
   const int lane = threadIdx.x & 31;
-  const int warps = (gridDim.x * blockDim.x) >> 5;
-  double wkl = 0.0;  // lane 0's share of sum_i w_i KL_i
-  for (int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; i < T; i += warps) {
-    const int r = pos[i];
-    float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
-    if (r >= 0 && n_vs > 0) {
-      float ms = -CUDART_INF_F, ss = 0.f, as = 0.f, mt = -CUDART_INF_F, st = 0.f;
+  const int g = threadIdx.x >> 5;
+  double wkl = 0.0;  // warp 0's share of sum_i w_i KL_i
+  const int n_row_blocks = (R + 31) / 32;
+  for (int rb = blockIdx.x; rb < n_row_blocks; rb += gridDim.x) {
+    const int r = rb * 32 + lane;
+    float ms = -CUDART_INF_F, ss = 0.f, as = 0.f, mt = -CUDART_INF_F, st = 0.f;
+    if (r < R) {
       // in a half-height tile, columns 128-255 of each split are a second partial at row r + 128
       const bool two = h0 >= 0 && r >= h0 && r < h0 + 128;
-      for (int j = lane; j < n_vs; j += 32) {
+#pragma unroll 4
+      for (int j = g; j < n_vs; j += kCombineGroups) {
         const float* b = part + (size_t)j * 5 * plane + r;
         merge_partial(ms, ss, as, mt, st, b[0], b[plane], b[2 * plane], b[3 * plane], b[4 * plane]);
         if (two)
           merge_partial(ms, ss, as, mt, st, b[128], b[plane + 128], b[2 * plane + 128], b[3 * plane + 128],
                         b[4 * plane + 128]);
       }
+    }
+    if (g > 0) {
+      sh[g - 1][0][lane] = ms;
+      sh[g - 1][1][lane] = ss;
+      sh[g - 1][2][lane] = as;
+      sh[g - 1][3][lane] = mt;
+      sh[g - 1][4][lane] = st;
+    }
+    __syncthreads();
+    if (g == 0 && r < R) {
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ms2 = __shfl_xor_sync(0xffffffffu, ms, o), ss2 = __shfl_xor_sync(0xffffffffu, ss, o);
-        const float as2 = __shfl_xor_sync(0xffffffffu, as, o), mt2 = __shfl_xor_sync(0xffffffffu, mt, o);
-        const float st2 = __shfl_xor_sync(0xffffffffu, st, o);
-        merge_partial(ms, ss, as, mt, st, ms2, ss2, as2, mt2, st2);
+      for (int k = 0; k < kCombineGroups - 1; ++k)
+        merge_partial(ms, ss, as, mt, st, sh[k][0][lane], sh[k][1][lane], sh[k][2][lane], sh[k][3][lane],
+                      sh[k][4][lane]);
+      const int i = idx ? idx[r] : r;
+      if (i >= 0 && i < T && pos[i] == r) {
+        float lse_s = 0.f, lse_t = 0.f, kl = 0.f;
+        if (n_vs > 0) {
+          const float ln2 = 0.69314718055994531f;
+          lse_s = (ms + log2f(ss)) * ln2;
+          lse_t = (mt + log2f(st)) * ln2;
+          kl = (as / ss) * ln2 - lse_s + lse_t;
+        }
+        kl_out[i] = kl;
+        stats[3 * (size_t)i + 0] = lse_s;
+        stats[3 * (size_t)i + 1] = lse_t;
+        stats[3 * (size_t)i + 2] = kl;
+        if (weights) wkl += (double)weights[i] * (double)kl;
       }
-      const float ln2 = 0.69314718055994531f;
-      lse_s = (ms + log2f(ss)) * ln2;
-      lse_t = (mt + log2f(st)) * ln2;
-      kl = (as / ss) * ln2 - lse_s + lse_t;
     }
-    if (lane == 0) {
-      kl_out[i] = kl;
-      stats[3 * (size_t)i + 0] = lse_s;
-      stats[3 * (size_t)i + 1] = lse_t;
-      stats[3 * (size_t)i + 2] = kl;
-      if (weights && r >= 0) wkl += (double)weights[i] * (double)kl;
-    }
+    __syncthreads();  // sh is rewritten by the next row block
   }
-  if (weights && lane == 0 && wkl != 0.0) atomicAdd(loss_acc, wkl);
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < T; i += gridDim.x * blockDim.x) {
+    if (pos[i] >= 0) continue;
+    kl_out[i] = 0.f;
+    stats[3 * (size_t)i + 0] = 0.f;
+    stats[3 * (size_t)i + 1] = 0.f;
+    stats[3 * (size_t)i + 2] = 0.f;
+  }
+  if (weights && g == 0) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) wkl += __shfl_xor_sync(0xffffffffu, wkl, o);
+    if (lane == 0 && wkl != 0.0) atomicAdd(loss_acc, wkl);
+  }
 }
 
 __global__ void k_bwd_rowc(const float* __restrict__ stats, const float* __restrict__ grad_kl,
@@ -289,11 +322,14 @@ cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
-                           float* kl_out, float* stats, const float* weights, double* loss_acc, int n_sm,
-                           cudaStream_t s) {
-  k_combine<<<grid_for((long)T * 32, n_sm, 256), 256, 0, s>>>(partials, pos, ctrl, T, T_pad, kl_out, stats,
-                                                               weights, loss_acc);
+cudaError_t launch_combine(const float* partials, const int32_t* pos, const int32_t* idx, const Ctrl* ctrl,
+                           int32_t T, int32_t T_pad, float* kl_out, float* stats, const float* weights,
+                           double* loss_acc, int n_sm, cudaStream_t s) {
+  // one block per 32 rows of T (an upper bound on the supervised rows), at most 8 per SM
+  long blocks = ((long)T + 31) / 32;
+  if (blocks > (long)n_sm * 8) blocks = (long)n_sm * 8;
+  k_combine<<<(int)(blocks < 1 ? 1 : blocks), 32 * kCombineGroups, 0, s>>>(partials, pos, idx, ctrl, T, T_pad,
+                                                                           kl_out, stats, weights, loss_acc);
   return cudaGetLastError();
 }
 

@@ -85,9 +85,10 @@ cudaError_t launch_compact(const uint8_t* mask, int32_t T, int32_t* idx, int32_t
 cudaError_t launch_gather_bf16(const void* H_s, const void* H_t, int32_t d_s, int32_t d_t, const int32_t* idx,
                                const Ctrl* ctrl, void* Hs_g, void* Ht_g, int32_t T_pad, int n_sm, cudaStream_t s);
 // weights != nullptr: also adds sum_i weights[i] KL_i to *loss_acc (the batch loss, fused here).
-cudaError_t launch_combine(const float* partials, const int32_t* pos, const Ctrl* ctrl, int32_t T, int32_t T_pad,
-                           float* kl_out, float* stats, const float* weights, double* loss_acc, int n_sm,
-                           cudaStream_t s);
+// idx maps gathered rows to token rows; nullptr: gathered row r is token row r.
+cudaError_t launch_combine(const float* partials, const int32_t* pos, const int32_t* idx, const Ctrl* ctrl,
+                           int32_t T, int32_t T_pad, float* kl_out, float* stats, const float* weights,
+                           double* loss_acc, int n_sm, cudaStream_t s);
 cudaError_t launch_bwd_rowc(const float* stats, const float* grad_kl, const int32_t* idx, const Ctrl* ctrl,
                             int32_t T_pad, float tau, float4* rowc, cudaStream_t s);
 cudaError_t launch_zero_rows(float* buf, int32_t cols, const Ctrl* ctrl, int32_t T_pad, int n_sm, cudaStream_t s);

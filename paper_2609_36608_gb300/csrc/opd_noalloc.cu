@@ -171,7 +171,7 @@ extern "C" opd_status opd_kl_forward_noalloc(const opd_problem* problem, const v
   fp.half_tile = 1;
   fp.vsplit = 0;
   if (launch_fused_forward(hs, ht, ws, wt, fp, sms, s) != cudaSuccess) return OPD_ERR_CUDA;
-  if (launch_combine(partials, pos, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
+  if (launch_combine(partials, pos, nullptr, ctrl, T, T_pad, kl_out, stats, nullptr, nullptr, sms, s) != cudaSuccess)
     return OPD_ERR_CUDA;
   k_noalloc_poison_on_timeout<<<1, 1024, 0, s>>>(kl_out, stats, T);
   if (cudaGetLastError() != cudaSuccess) return OPD_ERR_CUDA;
