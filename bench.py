@@ -413,6 +413,22 @@ def path_setup(path, w, lay, x, dev, opd_kl, world=1, rank=0):
     g = torch.Generator(device="cpu").manual_seed(w.seed)
     logp_teacher = (torch.randn(w.T, generator=g) - 7.0).to(dev)
     logp_old = (logp_teacher.cpu() + 0.3 * torch.randn(w.T, generator=g)).to(dev)
+    if world > 1:
+        # token-sharded data parallelism of the surrogate loss step, as for the reverse KL above
+        from paper_2609_36608_gb300 import data_parallel
+        n_local = int(lay.seg_id.max()) + 1
+        n_max = int(max_over_ranks(float(n_local), world, dev))
+        seg = np.where(lay.seg_id >= 0, lay.seg_id + rank * n_max, -1).astype(np.int32)
+        sharded = data_parallel.ShardedSurrogate(w.T, w.d_s, w.V, n_max * world, w.tau, device=dev)
+        dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
+        inputs = {"H_s": x["H_s"], "tokens": tokens, "logp_old": logp_old, "logp_teacher": logp_teacher,
+                  "mask": mask, "seg_id": torch.from_numpy(seg).to(dev)}
+
+        def step(i):
+            sharded.step(i["H_s"], x["W_s"], i["tokens"], i["logp_old"], i["logp_teacher"], i["mask"], i["seg_id"],
+                         dH, dW)
+        step.outputs = {"loss": sharded.loss_tok, "logp": sharded.logp, "dH": dH}
+        return inputs, step, sharded.loss, sharded.ws, 8.0 * R * w.V * w.d_s, 6.0 * R * w.V * w.d_s
     prob = opd_kl.make_problem(w.T, w.d_s, w.d_s, w.V, dtype, w.tau)
     ws = opd_kl.allocate_workspace(prob, dev)
     loss, logp = torch.empty(w.T, device=dev), torch.empty(w.T, device=dev)
@@ -710,8 +726,8 @@ def run_gpu(args):
         "config": {"workload": w.name, "T": w.T, "R": R, "R_all_ranks": R_job, "d_s": w.d_s, "d_t": w.d_t, "V": w.V,
                    "temperature": w.tau,
                    "parallelism": (f"dp{world}: token-sharded, one {w.T}-token batch per GPU, dW_s and the "
-                                   "loss all-reduced each step" if world > 1 and args.path == "kl" else
-                                   "replicas" if world > 1 else "single"),
+                                   "loss all-reduced each step" if world > 1 and args.path in ("kl", "surrogate")
+                                   else "replicas" if world > 1 else "single"),
                    "l2": "inputs larger than L2 (W_s + W_t = %.2f GB)" % ((w.d_s + w.d_t) * w.V * 2 / 1e9)},
         "tflops_executed": executed / (ms_step / 1000.0) / 1e12,
         "tflops_algorithmic": algorithmic / (ms_step / 1000.0) / 1e12,

@@ -25,6 +25,10 @@ calls and the collectives, on each rank's own buffers):
 The result on every rank equals one call over the whole batch (up to the order of the dW_s
 and L sums). A response may straddle two ranks: its rows' counts meet in step 2.
 
+ShardedSeqMeanKL runs these steps for the reverse KL. ShardedSurrogate runs them for the
+sampled-token dual-clip surrogate that the paper optimises (Appendix B.4), with
+opd_surrogate_fwd_bwd as step 4 and the per-token surrogate losses in step 5.
+
 The collectives are torch.distributed all-reduces (NCCL between GPUs, gloo on the CPU) on
 buffers the rank owns; no kernel of the library reads another GPU's memory.
 """
@@ -105,7 +109,40 @@ class Reducer:
         return works if async_op else []
 
 
-class ShardedSeqMeanKL:
+class _ShardedLoss:
+    """What the sharded loss steps share: the workspaces of the seq-mean-token-mean passes, the
+    histogram summed over the ranks, this rank's weights, and the sums of dW_s and of the loss."""
+
+    def __init__(self, T: int, n_ids: int, eps: float, device, group, bucket_bytes: int):
+        from . import opd_kl
+        self.lib = opd_kl
+        self.reducer = Reducer(group, bucket_bytes)
+        self.n_ids, self.eps, self.T = int(n_ids), float(eps), int(T)
+        dev = torch.device(device)
+        self.device = dev
+        self.seq_ws = torch.empty(opd_kl.opd_seq_mean_token_mean_workspace_size(self.n_ids), dtype=torch.uint8,
+                                  device=dev)
+        self.counts = torch.empty(2 * self.n_ids, dtype=torch.int32, device=dev)
+        self.weights = torch.empty(T, dtype=torch.float32, device=dev)
+        self.loss = torch.empty(1, dtype=torch.float32, device=dev)
+
+    def _weights(self, seg_id, mask) -> None:
+        """Steps 1-3: this rank's histogram, its sum over the ranks, this rank's weights."""
+        self.lib.opd_seq_mean_token_mean_counts(seg_id, mask, self.n_ids, self.counts, self.seq_ws)
+        self.reducer.sum_(self.counts)
+        self.lib.opd_seq_mean_token_mean_from_counts(seg_id, mask, self.n_ids, self.counts, self.eps, None,
+                                                     self.weights, None, self.seq_ws)
+
+    def _finish(self, seg_id, mask, per_token_loss, dW_s, reduce_grad: bool, async_grad: bool):
+        """Steps 5-6: this rank's part of L, then the sums of dW_s and L over the ranks."""
+        self.lib.opd_seq_mean_token_mean_from_counts(seg_id, mask, self.n_ids, self.counts, self.eps,
+                                                     per_token_loss, None, self.loss, self.seq_ws)
+        works = self.reducer.sum_rows_(dW_s, async_op=async_grad) if reduce_grad else []
+        self.reducer.sum_(self.loss)
+        return works
+
+
+class ShardedSeqMeanKL(_ShardedLoss):
     """The paper's batch loss over the per-token reverse KL and its gradients, for one rank's
     rows of a batch sharded by rows (see the module docstring for the steps).
 
@@ -118,21 +155,13 @@ class ShardedSeqMeanKL:
     def __init__(self, T: int, d_s: int, d_t: int, V: int, n_ids: int, temperature: float = 1.0,
                  eps: float = 1e-8, device="cuda", group=None, bucket_bytes: int = 256 << 20,
                  dtype: Optional[int] = None):
-        from . import opd_kl
-        self.lib = opd_kl
-        self.reducer = Reducer(group, bucket_bytes)
+        super().__init__(T, n_ids, eps, device, group, bucket_bytes)
+        opd_kl = self.lib
         dt = opd_kl.OPD_DTYPE_BF16 if dtype is None else dtype
         self.problem = opd_kl.make_problem(T, d_s, d_t, V, dt, temperature)
-        self.n_ids, self.eps, self.T = int(n_ids), float(eps), int(T)
-        dev = torch.device(device)
-        self.ws = opd_kl.allocate_workspace(self.problem, dev)
-        self.seq_ws = torch.empty(opd_kl.opd_seq_mean_token_mean_workspace_size(self.n_ids), dtype=torch.uint8,
-                                  device=dev)
-        self.counts = torch.empty(2 * self.n_ids, dtype=torch.int32, device=dev)
-        self.weights = torch.empty(T, dtype=torch.float32, device=dev)
-        self.kl = torch.empty(T, dtype=torch.float32, device=dev)
-        self.stats = torch.empty(T, 3, dtype=torch.float32, device=dev)
-        self.loss = torch.empty(1, dtype=torch.float32, device=dev)
+        self.ws = opd_kl.allocate_workspace(self.problem, self.device)
+        self.kl = torch.empty(T, dtype=torch.float32, device=self.device)
+        self.stats = torch.empty(T, 3, dtype=torch.float32, device=self.device)
 
     def step(self, H_s, H_t, W_s, W_t, mask, seg_id, dH_s, dW_s, accumulate_dW: bool = False,
              reduce_grad: bool = True, async_grad: bool = False):
@@ -144,15 +173,38 @@ class ShardedSeqMeanKL:
         Gradient accumulation over micro-batches: the sum over the ranks covers the whole dW_s
         buffer, earlier contents included, so pass accumulate_dW=True with reduce_grad=False for
         every micro-batch but the last, and reduce_grad=True (the default) with the last."""
-        lib = self.lib
-        lib.opd_seq_mean_token_mean_counts(seg_id, mask, self.n_ids, self.counts, self.seq_ws)
-        self.reducer.sum_(self.counts)
-        lib.opd_seq_mean_token_mean_from_counts(seg_id, mask, self.n_ids, self.counts, self.eps, None, self.weights,
-                                                None, self.seq_ws)
-        lib.opd_kl_fwd_bwd(self.problem, H_s, H_t, W_s, W_t, mask, self.weights, self.kl, self.stats, dH_s, dW_s,
-                           accumulate_dW, self.ws)
-        lib.opd_seq_mean_token_mean_from_counts(seg_id, mask, self.n_ids, self.counts, self.eps, self.kl, None,
-                                                self.loss, self.seq_ws)
-        works = self.reducer.sum_rows_(dW_s, async_op=async_grad) if reduce_grad else []
-        self.reducer.sum_(self.loss)
-        return works
+        self._weights(seg_id, mask)
+        self.lib.opd_kl_fwd_bwd(self.problem, H_s, H_t, W_s, W_t, mask, self.weights, self.kl, self.stats, dH_s,
+                                dW_s, accumulate_dW, self.ws)
+        return self._finish(seg_id, mask, self.kl, dW_s, reduce_grad, async_grad)
+
+
+class ShardedSurrogate(_ShardedLoss):
+    """The sampled-token dual-clip surrogate the paper optimises (Appendix B.4, Eq.
+    opd-token-advantage, opd-ratio, opd-dual-clip, opd-surrogate) under the same row sharding:
+    the seq-mean-token-mean weights of the whole batch from the summed histogram, this rank's
+    opd_surrogate_fwd_bwd with those weights, then the sums of dW_s and of L over the ranks.
+    T is this rank's row count; d and V are the student head's sizes; `params` holds the
+    surrogate's constants (None: the paper's delta = 0.2, kappa = 3, clip 20). The teacher
+    enters only through logp_teacher, scored beforehand (opd_score_tokens)."""
+
+    def __init__(self, T: int, d: int, V: int, n_ids: int, temperature: float = 1.0, eps: float = 1e-8,
+                 device="cuda", group=None, bucket_bytes: int = 256 << 20, params=None):
+        super().__init__(T, n_ids, eps, device, group, bucket_bytes)
+        opd_kl = self.lib
+        self.problem = opd_kl.make_problem(T, d, d, V, opd_kl.OPD_DTYPE_BF16, temperature)
+        self.ws = opd_kl.allocate_workspace(self.problem, self.device)
+        self.params = params
+        self.loss_tok = torch.empty(T, dtype=torch.float32, device=self.device)
+        self.logp = torch.empty(T, dtype=torch.float32, device=self.device)
+
+    def step(self, H_s, W_s, tokens, logp_old, logp_teacher, mask, seg_id, dH_s, dW_s, accumulate_dW: bool = False,
+             reduce_grad: bool = True, async_grad: bool = False):
+        """Writes this rank's per-token losses (self.loss_tok) and log-probabilities (self.logp),
+        its dH_s rows and, summed over every rank, dW_s and L (self.loss[0]). accumulate_dW,
+        reduce_grad and async_grad as for ShardedSeqMeanKL.step."""
+        self._weights(seg_id, mask)
+        self.lib.opd_surrogate_fwd_bwd(self.problem, H_s, W_s, tokens, logp_old, logp_teacher, mask, self.weights,
+                                       self.loss_tok, self.logp, dH_s, dW_s, accumulate_dW, self.ws,
+                                       params=self.params)
+        return self._finish(seg_id, mask, self.loss_tok, dW_s, reduce_grad, async_grad)

@@ -4,8 +4,8 @@ The rank takes its contiguous rows of one small packed batch (row_shards), build
 histogram of response ids (standing in for the device pass opd_seq_mean_token_mean_counts),
 sums it over the ranks with the library's Reducer, computes its rows' KL, dH_s and dW_s part
 with the float64 oracle under the whole batch's seq-mean-token-mean weights, and sums dW_s
-(in several buckets) and its part of the loss over the ranks. The parent test compares the
-result with one oracle call over the whole batch."""
+(in several buckets) and its part of the loss over the ranks; then the same for the dual-clip
+surrogate. The parent test compares the results with one oracle call over the whole batch."""
 
 import os
 import sys
@@ -26,6 +26,16 @@ def batch():
     w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="dp_small", T=300, d_s=32, d_t=48, V=200, tau=0.8,
                      n_traj=3, traj_len=100, seed=5)
     return w, synth.layout(w)
+
+
+def surrogate_inputs(w):
+    """Sampled tokens and behaviour / teacher log-probabilities: the log-ratios spread over the
+    ratio clip and the advantages take both signs."""
+    rng = np.random.default_rng(7)
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    logp_teacher = rng.normal(-6.0, 1.0, w.T)
+    logp_old = logp_teacher + rng.normal(0.0, 1.0, w.T)
+    return tokens, logp_old, logp_teacher
 
 
 def main():
@@ -52,8 +62,17 @@ def main():
         work.wait()
     loss = torch.tensor([float(np.sum(g[rows] * res.kl))], dtype=torch.float64)
     red.sum_(loss)
+    # the dual-clip surrogate under the same sharding (its per-token losses weighted alike)
+    tokens, logp_old, logp_teacher = surrogate_inputs(w)
+    sres = oracle.surrogate(host[0], host[2], tokens, logp_old, logp_teacher, lay.mask, g, w.tau, rows=rows,
+                            n_threads=1)
+    sdW = torch.from_numpy(np.ascontiguousarray(sres.dW_s))
+    red.sum_rows_(sdW)
+    sloss = torch.tensor([float(np.sum(g[rows] * sres.loss))], dtype=torch.float64)
+    red.sum_(sloss)
     np.savez(os.path.join(os.environ["OPD_TEST_OUT"], f"rank{rank}.npz"), lo=lo, hi=hi, counts=counts.numpy(),
-             kl=res.kl, dH=res.dH_s, dW=dW.numpy(), loss=loss.numpy(), buckets=len(red.buckets(w.V, w.d_s * 8)))
+             kl=res.kl, dH=res.dH_s, dW=dW.numpy(), loss=loss.numpy(), buckets=len(red.buckets(w.V, w.d_s * 8)),
+             s_loss_tok=sres.loss, s_dH=sres.dH_s, s_dW=sdW.numpy(), s_loss=sloss.numpy())
     dist.destroy_process_group()
 
 

@@ -1,6 +1,7 @@
 """Token-sharded data parallelism (the paper trains the student on two GPUs, Appendix C) on
-the CPU: the row partition, the collectives' bucketing, and two gloo ranks whose sharded step,
-computed with the float64 oracle, equals one oracle call over the whole batch."""
+the CPU: the row partition, the collectives' bucketing, and two gloo ranks whose sharded steps
+(the reverse KL and the dual-clip surrogate), computed with the float64 oracle, equal one oracle
+call over the whole batch."""
 
 import os
 import socket
@@ -85,3 +86,12 @@ def test_two_gloo_ranks_equal_one_whole_batch_oracle_call(tmp_path, oracle_mod):
         assert int(r[k]["buckets"]) > 1
         np.testing.assert_allclose(r[k]["dW"], whole.dW_s, rtol=1e-12, atol=1e-15)
         np.testing.assert_allclose(r[k]["loss"][0], float(np.sum(g * whole.kl)), rtol=1e-12)
+    # the dual-clip surrogate under the same split
+    tokens, logp_old, logp_teacher = dp_worker.surrogate_inputs(w)
+    sw = oracle_mod.surrogate(host[0], host[2], tokens, logp_old, logp_teacher, lay.mask, g, w.tau)
+    np.testing.assert_array_equal(np.concatenate([r[0]["s_loss_tok"], r[1]["s_loss_tok"]]), sw.loss)
+    np.testing.assert_array_equal(np.concatenate([r[0]["s_dH"], r[1]["s_dH"]]), sw.dH_s)
+    assert np.abs(sw.dH_s).max() > 0  # some tokens inside the clip carry a gradient
+    for k in range(2):
+        np.testing.assert_allclose(r[k]["s_dW"], sw.dW_s, rtol=1e-12, atol=1e-15)
+        np.testing.assert_allclose(r[k]["s_loss"][0], float(np.sum(g * sw.loss)), rtol=1e-12)

@@ -211,3 +211,98 @@ def test_shards_with_no_rows_and_loss_only_requests(lib, oracle_mod):
     want = float(np.sum(ref * loss_in.cpu().numpy().astype(np.float64)))
     assert abs(p.sum() - want) <= 1e-6 * abs(want)
     assert dp.row_shards(w.T, 3, np.zeros(w.T, np.uint8)) == [(0, 0), (0, 0), (0, w.T)]
+
+
+def _off_kinks(seed, n):
+    """Log-ratio offsets in [-0.6, 1.4] at least 0.02 from the ratio clip's kinks (ln 0.8, ln 1.2)
+    and the dual clip's (ln 3), so that fp32 and fp64 take the same branch."""
+    edges = np.log([0.8, 1.2, 3.0])
+    rng = np.random.default_rng(seed)
+    out = rng.uniform(-0.6, 1.4, 4 * n)
+    out = out[np.min(np.abs(out[:, None] - edges[None, :]), axis=1) > 0.02]
+    return out[:n]
+
+
+@pytest.mark.parametrize("world", [1, 2, 3])
+def test_sharded_surrogate_equals_the_whole_batch(lib, oracle_mod, world):
+    """ShardedSurrogate's calls per shard (with one shard: its step itself); the shards' dW_s
+    parts and losses summed as the all-reduce sums them, against the float64 oracle's surrogate
+    over the whole batch under the whole batch's seq-mean-token-mean weights."""
+    from paper_2609_36608_gb300 import data_parallel as dp
+    w, lay = _batch(name="dp_sur", T=900, d_s=160, V=1300, n_traj=3, seed=65)
+    x = synth.hidden_and_heads(w, "cuda")
+    Hs, Ws = synth.host_values(x["H_s"]), synth.host_values(x["W_s"])
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    _, lp_ref = oracle_mod.score(Hs, Ws, tokens, w.tau)
+    logp_old = (lp_ref - _off_kinks(world, w.T)).astype(np.float32)
+    adv = np.random.default_rng(9).choice([-1.0, 1.0], w.T) * np.random.default_rng(10).uniform(0.2, 1.5, w.T)
+    logp_teacher = (logp_old.astype(np.float64) + adv).astype(np.float32)
+    n_ids = int(lay.seg_id.max()) + 1
+    f32 = lambda a: torch.from_numpy(np.asarray(a, np.float32)).cuda()
+    seg, mask = torch.from_numpy(lay.seg_id).cuda(), torch.from_numpy(lay.mask).cuda()
+    tok, lo_t, lt_t = torch.from_numpy(tokens).cuda(), f32(logp_old), f32(logp_teacher)
+    shards = dp.row_shards(w.T, world, lay.mask)
+    steps = [dp.ShardedSurrogate(hi - lo, w.d_s, w.V, n_ids, w.tau) for lo, hi in shards]
+    dH = torch.full((w.T, w.d_s), float("nan"), device="cuda")
+    dWs = [torch.full((w.V, w.d_s), float("nan"), device="cuda") for _ in shards]
+    loss_tok = torch.empty(w.T, device="cuda")
+    if world == 1:
+        steps[0].step(x["H_s"], x["W_s"], tok, lo_t, lt_t, mask, seg, dH, dWs[0])
+        loss, dW = steps[0].loss, dWs[0]
+        loss_tok.copy_(steps[0].loss_tok)
+    else:
+        for st, (lo, hi) in zip(steps, shards):
+            lib.opd_seq_mean_token_mean_counts(seg[lo:hi], mask[lo:hi], n_ids, st.counts, st.seq_ws)
+        total = sum(st.counts for st in steps)
+        loss = torch.zeros(1, device="cuda")
+        for st, (lo, hi), dW_k in zip(steps, shards, dWs):
+            st.counts.copy_(total)
+            args = (seg[lo:hi], mask[lo:hi], n_ids, st.counts, st.eps)
+            lib.opd_seq_mean_token_mean_from_counts(*args, None, st.weights, None, st.seq_ws)
+            lib.opd_surrogate_fwd_bwd(st.problem, x["H_s"][lo:hi], x["W_s"], tok[lo:hi], lo_t[lo:hi], lt_t[lo:hi],
+                                      mask[lo:hi], st.weights, st.loss_tok, st.logp, dH[lo:hi], dW_k, False, st.ws)
+            lib.opd_seq_mean_token_mean_from_counts(*args, st.loss_tok, None, st.loss, st.seq_ws)
+            loss_tok[lo:hi] = st.loss_tok
+            loss += st.loss
+        dW = sum(dWs)
+    torch.cuda.synchronize()
+    for st in steps:
+        assert lib.opd_kl_get_status(st.ws) == lib.OPD_OK and lib.opd_kl_get_status(st.seq_ws) == lib.OPD_OK
+    g = oracle_mod.seq_mean_token_mean_weights(lay.seg_id, lay.mask)
+    ref = oracle_mod.surrogate(Hs, Ws, tokens, logp_old.astype(np.float64), logp_teacher.astype(np.float64),
+                               lay.mask, g.astype(np.float32).astype(np.float64), w.tau)
+    got = loss_tok.cpu().numpy().astype(np.float64)
+    assert (np.abs(got - ref.loss) <= 1e-4 + 2e-3 * np.abs(ref.loss)).all()
+    assert _rel(dH.cpu().numpy(), ref.dH_s) <= GRAD_REL
+    assert _rel(dW.cpu().numpy(), ref.dW_s) <= GRAD_REL
+    want = float(np.sum(g * ref.loss))
+    assert abs(float(loss[0]) - want) <= 1e-4 * abs(want) + 1e-7
+
+
+def test_bench_data_parallel_surrogate_step_in_a_process_group_of_one(lib, tmp_path):
+    """bench.py's N > 1 surrogate step (ShardedSurrogate with global response ids) as rank 0 of
+    a one-rank NCCL group equals the single-GPU surrogate loss step of the same batch."""
+    import torch.distributed as dist
+    import bench
+    w, lay = _batch(name="dp_bench_sur", T=1200, n_traj=4, seed=66)
+    x = synth.hidden_and_heads(w, "cuda")
+    dev = torch.device("cuda", torch.cuda.current_device())
+    dist.init_process_group("nccl", init_method=f"file://{tmp_path}/pg", world_size=1, rank=0)
+    try:
+        inputs, step, result, ws, _, _ = bench.path_setup("surrogate", w, lay, x, dev, lib, world=2, rank=0)
+        step(inputs)
+        torch.cuda.synchronize()
+        assert lib.opd_kl_get_status(ws) == lib.OPD_OK
+        dp_loss = float(result[0])
+        dp_tok = step.outputs["loss"].cpu().numpy()
+        dp_dH = step.outputs["dH"].cpu().numpy()
+    finally:
+        dist.destroy_process_group()
+    inputs1, step1, result1, ws1, _, _ = bench.path_setup("surrogate", w, lay, x, dev, lib)
+    step1(inputs1)
+    torch.cuda.synchronize()
+    assert lib.opd_kl_get_status(ws1) == lib.OPD_OK
+    np.testing.assert_array_equal(dp_tok, step1.outputs["loss"].cpu().numpy())
+    assert _rel(dp_dH, step1.outputs["dH"].cpu().numpy().astype(np.float64)) < 1e-5
+    ref = float(result1[0])
+    assert abs(dp_loss - ref) <= 1e-6 * abs(ref) + 1e-9
