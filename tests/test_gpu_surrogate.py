@@ -405,3 +405,19 @@ def test_surrogate_loss_step_in_a_cuda_graph(lib):
     # dH_s: split-K partial sums in arrival order; L: a double sum over blocks in arrival order
     assert _rel(dH.cpu().numpy(), eager["dH"].cpu().numpy().astype(np.float64)) < 1e-5
     assert np.isfinite(total.item()) and abs(total.item() - eager["total"].item()) <= 1e-6 * abs(eager["total"].item())
+
+
+def test_surrogate_and_scoring_with_every_row_masked(lib):
+    """R = 0 with T > 0: zeros out, dW_s zeroed (or left as it was when accumulating), status OK."""
+    w = _case(T=300, d_s=64, V=700, n_traj=3, traj_len=100, seed=44)
+    x = synth.hidden_and_heads(w, "cuda")
+    tokens = synth.token_ids(w.seed, w.T, w.V)
+    mask = np.zeros(w.T, np.uint8)
+    lse, lp = _score(lib, w, x["H_s"], x["W_s"], tokens, mask)
+    assert (lse == 0).all() and (lp == 0).all()
+    zeros = np.zeros(w.T, np.float32)
+    loss, lp2, dH, dW = _surrogate(lib, w, x, tokens, zeros - 5.0, zeros - 4.0, mask, zeros + 1.0)
+    assert (loss == 0).all() and (lp2 == 0).all() and (dH == 0).all() and (dW == 0).all()
+    init = torch.full((w.V, w.d_s), 3.0, device="cuda")
+    _, _, _, dW2 = _surrogate(lib, w, x, tokens, zeros - 5.0, zeros - 4.0, mask, zeros + 1.0, True, init)
+    assert (dW2 == 3.0).all()
