@@ -356,13 +356,10 @@ def path_setup(path, w, lay, x, dev, opd_kl, world=1, rank=0):
         # token-sharded data parallelism: this rank's batch, the paper's batch loss over every
         # rank's rows (response ids made global), dW_s and L summed over the ranks each step
         from paper_2609_36608_gb300 import data_parallel
-        n_local = int(lay.seg_id.max()) + 1
-        n_max = int(max_over_ranks(float(n_local), world, dev))
-        seg = np.where(lay.seg_id >= 0, lay.seg_id + rank * n_max, -1).astype(np.int32)
-        sharded = data_parallel.ShardedSeqMeanKL(w.T, w.d_s, w.d_t, w.V, n_max * world, w.tau, device=dev,
-                                                 dtype=dtype)
+        seg, n_ids = data_parallel.global_response_ids(torch.from_numpy(lay.seg_id).to(dev))
+        sharded = data_parallel.ShardedSeqMeanKL(w.T, w.d_s, w.d_t, w.V, n_ids, w.tau, device=dev, dtype=dtype)
         dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
-        inputs = {"H_s": x["H_s"], "H_t": x["H_t"], "mask": mask, "seg_id": torch.from_numpy(seg).to(dev)}
+        inputs = {"H_s": x["H_s"], "H_t": x["H_t"], "mask": mask, "seg_id": seg}
 
         def step(i):
             sharded.step(i["H_s"], i["H_t"], x["W_s"], x["W_t"], i["mask"], i["seg_id"], dH, dW)
@@ -416,13 +413,11 @@ def path_setup(path, w, lay, x, dev, opd_kl, world=1, rank=0):
     if world > 1:
         # token-sharded data parallelism of the surrogate loss step, as for the reverse KL above
         from paper_2609_36608_gb300 import data_parallel
-        n_local = int(lay.seg_id.max()) + 1
-        n_max = int(max_over_ranks(float(n_local), world, dev))
-        seg = np.where(lay.seg_id >= 0, lay.seg_id + rank * n_max, -1).astype(np.int32)
-        sharded = data_parallel.ShardedSurrogate(w.T, w.d_s, w.V, n_max * world, w.tau, device=dev)
+        seg, n_ids = data_parallel.global_response_ids(torch.from_numpy(lay.seg_id).to(dev))
+        sharded = data_parallel.ShardedSurrogate(w.T, w.d_s, w.V, n_ids, w.tau, device=dev)
         dH, dW = torch.empty(w.T, w.d_s, device=dev), torch.empty(w.V, w.d_s, device=dev)
         inputs = {"H_s": x["H_s"], "tokens": tokens, "logp_old": logp_old, "logp_teacher": logp_teacher,
-                  "mask": mask, "seg_id": torch.from_numpy(seg).to(dev)}
+                  "mask": mask, "seg_id": seg}
 
         def step(i):
             sharded.step(i["H_s"], x["W_s"], i["tokens"], i["logp_old"], i["logp_teacher"], i["mask"], i["seg_id"],

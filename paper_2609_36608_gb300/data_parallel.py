@@ -67,6 +67,24 @@ def row_shards(T: int, world: int, mask: Optional[Sequence[int]] = None) -> List
     return [(cuts[k], cuts[k + 1]) for k in range(world)]
 
 
+def global_response_ids(seg_id: torch.Tensor, group=None):
+    """Response ids made global across the ranks, for batches whose responses each live on one
+    rank (every rank packs its own batch, as under the paper's per-GPU token budget).
+
+    Rank k's ids b >= 0 become b + k n_max, with n_max the largest local id count over the
+    ranks (ids < 0, rows outside every response, stay as they are). Returns the new ids (same
+    device and dtype) and the global id count n_max * world. One all-reduce of one integer;
+    with no process group (or one rank) the ids come back unchanged."""
+    n_local = int(seg_id.max().item()) + 1 if seg_id.numel() else 0
+    if not _active(group):
+        return seg_id.clone(), max(n_local, 1)
+    t = torch.tensor([n_local], dtype=torch.int64, device=seg_id.device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX, group=group)
+    n_max = max(int(t.item()), 1)
+    rank, world = dist.get_rank(group), dist.get_world_size(group)
+    return torch.where(seg_id >= 0, seg_id + rank * n_max, seg_id), n_max * world
+
+
 def _active(group) -> bool:
     return dist.is_available() and dist.is_initialized() and dist.get_world_size(group) > 1
 

@@ -70,7 +70,11 @@ def main():
     red.sum_rows_(sdW)
     sloss = torch.tensor([float(np.sum(g[rows] * sres.loss))], dtype=torch.float64)
     red.sum_(sloss)
+    # global ids for batches packed per rank: rank k holds 3 + k local responses
+    local = torch.tensor([-1, 0, 0, 1, -1, 2 + rank], dtype=torch.int32)
+    gids, n_ids_all = dp.global_response_ids(local)
     np.savez(os.path.join(os.environ["OPD_TEST_OUT"], f"rank{rank}.npz"), lo=lo, hi=hi, counts=counts.numpy(),
+             gids=gids.numpy(), n_ids_all=n_ids_all,
              kl=res.kl, dH=res.dH_s, dW=dW.numpy(), loss=loss.numpy(), buckets=len(red.buckets(w.V, w.d_s * 8)),
              s_loss_tok=sres.loss, s_dH=sres.dH_s, s_dW=sdW.numpy(), s_loss=sloss.numpy())
     dist.destroy_process_group()

@@ -86,6 +86,10 @@ def test_two_gloo_ranks_equal_one_whole_batch_oracle_call(tmp_path, oracle_mod):
         assert int(r[k]["buckets"]) > 1
         np.testing.assert_allclose(r[k]["dW"], whole.dW_s, rtol=1e-12, atol=1e-15)
         np.testing.assert_allclose(r[k]["loss"][0], float(np.sum(g * whole.kl)), rtol=1e-12)
+    # global response ids: n_max = 4 (rank 1's ids reach 3), so rank k's ids shift by 4 k
+    assert int(r[0]["n_ids_all"]) == 8 and int(r[1]["n_ids_all"]) == 8
+    np.testing.assert_array_equal(r[0]["gids"], [-1, 0, 0, 1, -1, 2])
+    np.testing.assert_array_equal(r[1]["gids"], [-1, 4, 4, 5, -1, 7])
     # the dual-clip surrogate under the same split
     tokens, logp_old, logp_teacher = dp_worker.surrogate_inputs(w)
     sw = oracle_mod.surrogate(host[0], host[2], tokens, logp_old, logp_teacher, lay.mask, g, w.tau)
