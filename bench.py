@@ -140,7 +140,8 @@ class ClockSampler:
         reasons = sorted({names[i] for r in rows for i in range(4) if r[4 + i].lower().startswith("active")})
         pw = [float(r[2]) for r in rows if re.match(r"^[\d.]+$", r[2])]
         return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None}
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(pw) if pw else None,
+                "power_w_median": float(np.median(pw)) if pw else None}
 
 
 def choose_peak(clocks, peaks, peak_src):
