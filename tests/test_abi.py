@@ -224,3 +224,18 @@ def test_binding_checks_every_buffer_before_the_call(lib):
     f32p = lib.make_problem(T, d_s, d_t, V, lib.OPD_DTYPE_F32, 1.0)
     with pytest.raises(TypeError, match="H_s: dtype torch.bfloat16"):
         lib.opd_kl_forward(f32p, good["H_s"], f32(T, d_t), f32(V, d_s), f32(V, d_t), mask, f32(T), f32(T, 3), ws)
+
+
+def test_row_chunk_sizing_for_a_workspace_budget(lib):
+    from paper_2609_36608_gb300 import chunking
+    p = lib.make_problem(16384, 2048, 4096, 151936, lib.OPD_DTYPE_BF16, 1.0)
+    full = lib.opd_kl_workspace_size(p)
+    assert chunking.max_rows_for_workspace(p, full) == 16384
+    for budget in (1 << 30, 2 << 30, full - 1):
+        rows = chunking.max_rows_for_workspace(p, budget)
+        assert rows % 256 == 0 and 0 < rows < 16384
+        fits = lambda r: lib.opd_kl_workspace_size(lib.make_problem(r, 2048, 4096, 151936, 0, 1.0)) <= budget
+        assert fits(rows) and not fits(rows + 256)
+    assert chunking.max_rows_for_workspace(p, 1 << 20) == 0
+    small = lib.make_problem(100, 64, 64, 500, lib.OPD_DTYPE_BF16, 1.0)
+    assert chunking.max_rows_for_workspace(small, lib.opd_kl_workspace_size(small)) == 100

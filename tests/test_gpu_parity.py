@@ -600,3 +600,36 @@ def test_full_size_sampled_rows(lib, oracle_mod, name):
     ref2 = oracle_mod.opd_kl(H_s, H_t, W_s, W_t, mask2, _g64(g, mask2), w.tau, rows=sub, want_dH=False)
     assert _rel(out2["dW"], ref2.dW_s) <= GRAD_REL, _rel(out2["dW"], ref2.dW_s)
     _check_kl(out2["kl"][sub], ref2.kl)
+
+
+def test_row_chunk_helper_under_a_workspace_budget(lib, oracle_mod):
+    """kl_fwd_bwd_in_row_chunks with a budget that holds 256 rows: four chunks of one shared
+    workspace, against one call and against the oracle; with accumulate_dW the first chunk adds
+    to dW_s too."""
+    from paper_2609_36608_gb300 import chunking
+    w = _small_bf16(T=900, V=2000, seed=32)
+    lay = synth.layout(w)
+    g = synth.uniform_weights(w.seed, w.T)
+    x = synth.hidden_and_heads(w, "cuda")
+    whole = _run(lib, w, x, lay.mask, g)
+    prob = lib.make_problem(w.T, w.d_s, w.d_t, w.V, lib.OPD_DTYPE_BF16, w.tau)
+    budget = lib.opd_kl_workspace_size(lib.make_problem(256, w.d_s, w.d_t, w.V, lib.OPD_DTYPE_BF16, w.tau))
+    assert chunking.max_rows_for_workspace(prob, budget) == 256
+    mask = torch.from_numpy(lay.mask).cuda()
+    grad = torch.from_numpy(np.asarray(g, np.float32)).cuda()
+    kl, stats = torch.full((w.T,), float("nan"), device="cuda"), torch.full((w.T, 3), float("nan"), device="cuda")
+    dH = torch.full((w.T, w.d_s), float("nan"), device="cuda")
+    init = torch.randn(w.V, w.d_s, device="cuda", generator=torch.Generator("cuda").manual_seed(3))
+    dW = init.clone()
+    n = chunking.kl_fwd_bwd_in_row_chunks(prob, x["H_s"], x["H_t"], x["W_s"], x["W_t"], mask, grad, kl, stats, dH,
+                                          dW, True, budget)
+    torch.cuda.synchronize()
+    assert n == 4
+    got_kl = kl.cpu().numpy()
+    np.testing.assert_allclose(got_kl, whole["kl"], rtol=1e-6, atol=1e-7)
+    assert _rel(dH.cpu().numpy(), whole["dH"].astype(np.float64)) < 1e-5
+    assert _rel((dW - init).cpu().numpy(), whole["dW"].astype(np.float64)) < 1e-5
+    ref = oracle_mod.opd_kl(*_host(x), lay.mask, _g64(g, lay.mask), w.tau)
+    _check_kl(got_kl, ref.kl)
+    assert _rel(dH.cpu().numpy(), ref.dH_s) <= GRAD_REL
+    assert _rel((dW - init).cpu().numpy(), ref.dW_s) <= GRAD_REL
