@@ -306,3 +306,68 @@ def test_bench_data_parallel_surrogate_step_in_a_process_group_of_one(lib, tmp_p
     assert _rel(dp_dH, step1.outputs["dH"].cpu().numpy().astype(np.float64)) < 1e-5
     ref = float(result1[0])
     assert abs(dp_loss - ref) <= 1e-6 * abs(ref) + 1e-9
+
+
+def _random_dp_cases(n, seed=977):
+    rng = np.random.default_rng(seed)
+    out = []
+    for i in range(n):
+        T = int(rng.integers(1, 700))
+        out.append(dict(T=T, d_s=8 * int(rng.integers(1, 33)), d_t=8 * int(rng.integers(1, 49)),
+                        V=int(rng.integers(2, 3000)), tau=float(rng.choice([0.5, 1.0, 1.6])),
+                        world=int(rng.integers(2, 6)), density=float(rng.uniform(0.0, 1.0)),
+                        n_resp=int(rng.integers(1, 12)), seed=300 + i))
+    return out
+
+
+@pytest.mark.parametrize("case", _random_dp_cases(6), ids=lambda c: f"T{c['T']}-w{c['world']}-V{c['V']}")
+def test_sharded_kl_random_shapes(lib, oracle_mod, case):
+    """Seeded random problems split over 2-5 emulated ranks: random masks (density 0-1, so some
+    shards may hold no supervised row) and random response layouts (responses straddle cuts). The
+    summed dW_s and loss and the per-row KL and dH_s match the whole-batch oracle."""
+    from paper_2609_36608_gb300 import data_parallel as dp
+    rng = np.random.default_rng(case["seed"])
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="dp_rand", T=case["T"], d_s=case["d_s"], d_t=case["d_t"],
+                     V=case["V"], tau=case["tau"], n_traj=1, traj_len=case["T"], seed=case["seed"])
+    mask = (rng.random(w.T) < case["density"]).astype(np.uint8)
+    seg = np.sort(rng.integers(-1, case["n_resp"], w.T)).astype(np.int32)
+    n_ids = case["n_resp"]
+    x = synth.hidden_and_heads(w, "cuda")
+    seg_t, mask_t = torch.from_numpy(seg).cuda(), torch.from_numpy(mask).cuda()
+    shards = dp.row_shards(w.T, case["world"], mask)
+    steps = [dp.ShardedSeqMeanKL(hi - lo, w.d_s, w.d_t, w.V, n_ids, w.tau) for lo, hi in shards]
+    for st, (lo, hi) in zip(steps, shards):
+        lib.opd_seq_mean_token_mean_counts(seg_t[lo:hi], mask_t[lo:hi], n_ids, st.counts, st.seq_ws)
+    total = sum(st.counts for st in steps)
+    dH = torch.full((w.T, w.d_s), float("nan"), device="cuda")
+    kl = torch.empty(w.T, device="cuda")
+    dW = torch.zeros(w.V, w.d_s, device="cuda")
+    loss = torch.zeros(1, device="cuda")
+    for st, (lo, hi) in zip(steps, shards):
+        st.counts.copy_(total)
+        args = (seg_t[lo:hi], mask_t[lo:hi], n_ids, st.counts, st.eps)
+        lib.opd_seq_mean_token_mean_from_counts(*args, None, st.weights, None, st.seq_ws)
+        dW_k = torch.empty(w.V, w.d_s, device="cuda")
+        lib.opd_kl_fwd_bwd(st.problem, x["H_s"][lo:hi], x["H_t"][lo:hi], x["W_s"], x["W_t"], mask_t[lo:hi],
+                           st.weights, st.kl, st.stats, dH[lo:hi], dW_k, False, st.ws)
+        lib.opd_seq_mean_token_mean_from_counts(*args, st.kl, None, st.loss, st.seq_ws)
+        kl[lo:hi] = st.kl
+        dW += dW_k
+        loss += st.loss
+    torch.cuda.synchronize()
+    for st in steps:
+        assert lib.opd_kl_get_status(st.ws) == lib.OPD_OK and lib.opd_kl_get_status(st.seq_ws) == lib.OPD_OK
+    g = oracle_mod.seq_mean_token_mean_weights(seg, mask)
+    ref = oracle_mod.opd_kl(*(synth.host_values(x[k]) for k in ("H_s", "H_t", "W_s", "W_t")), mask,
+                            g.astype(np.float32).astype(np.float64), w.tau)
+    got = kl.cpu().numpy().astype(np.float64)
+    assert (np.abs(got - ref.kl) <= KL_ABS + KL_REL * np.abs(ref.kl)).all()
+    sup = mask != 0
+    assert (dH.cpu().numpy()[~sup] == 0).all()
+    if sup.any():
+        assert _rel(dH.cpu().numpy(), ref.dH_s) <= GRAD_REL
+        assert _rel(dW.cpu().numpy(), ref.dW_s) <= GRAD_REL
+    else:
+        assert (dW == 0).all()
+    want = float(np.sum(g * ref.kl))
+    assert abs(float(loss[0]) - want) <= 1e-4 * abs(want) + 1e-7
