@@ -704,6 +704,11 @@ def run_gpu(args):
                     "frac_of_sustained": achieved / peaks["bf16_tflops_sustained"],
                     # the same kernel at its kernel-pass share of the timed region's step time
                     "frac_at_timed_step": achieved / peak * ms_profiled / ms_step,
+                    # per clock: scaled to the clock the sustained peak was measured at (when both are known)
+                    "frac_sustained_per_clock": (achieved / peaks["bf16_tflops_sustained"] * peaks["sustained_mhz"]
+                                                 / clocks_kernel_pass["sm_mhz"])
+                    if clocks_kernel_pass and clocks_kernel_pass.get("sm_mhz") and peaks.get("sustained_mhz")
+                    else None,
                     "algorithmic_flops_per_launch": per_launch}
 
     cpu, parity = None, None
