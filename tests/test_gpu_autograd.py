@@ -110,3 +110,36 @@ def test_surrogate_loss_autograd_and_scoring(mods, oracle_mod):
     assert abs(float(loss.detach()) - want) <= 1e-4 + 2e-3 * abs(want)
     assert _rel(H_s.grad.float().cpu().numpy(), ref.dH_s) <= 1e-2
     assert _rel(W_s.grad.float().cpu().numpy(), ref.dW_s) <= 1e-2
+
+
+def test_debug_mode_raises_on_bad_ids_through_autograd(mods, monkeypatch):
+    """The autograd functions do not read the device status word; with OPD_KL_SYNC_CHECK=1 the
+    library itself synchronises after each call and the binding raises OpdError. A token id past
+    the vocabulary (scoring) and a response id past n_ids (the surrogate's weights) are reported
+    that way; without debug mode the same calls return."""
+    ag, lib = mods
+    w = synth.scaled(synth.WORKLOADS["qwen3_1p7b"], name="dbg", T=256, d_s=64, d_t=64, V=500, tau=1.0,
+                     n_traj=2, traj_len=128, seed=53)
+    lay = synth.layout(w)
+    x = synth.hidden_and_heads(w, "cuda")
+    mask = torch.from_numpy(lay.mask).cuda()
+    tokens = torch.from_numpy(synth.token_ids(w.seed, w.T, w.V)).cuda()
+    bad_tokens = tokens.clone()
+    bad_tokens[int(np.flatnonzero(lay.mask)[0])] = w.V + 3
+    seg = torch.from_numpy(lay.seg_id).cuda()
+    n_ids = int(lay.seg_id.max()) + 1
+    bad_seg = seg.clone()
+    bad_seg[int(np.flatnonzero(lay.seg_id >= 0)[0])] = n_ids + 5
+    lp = torch.full((w.T,), -6.0, device="cuda")
+    ag.score_tokens(x["H_s"], x["W_s"], bad_tokens, mask)  # outside debug mode: returns
+    ag.OPDSurrogateLoss.apply(x["H_s"], x["W_s"], tokens, lp, lp + 0.5, mask, bad_seg, n_ids, 1.0, 1e-8)
+    torch.cuda.synchronize()
+    monkeypatch.setenv("OPD_KL_SYNC_CHECK", "1")
+    with pytest.raises(lib.OpdError) as e1:
+        ag.score_tokens(x["H_s"], x["W_s"], bad_tokens, mask)
+    assert e1.value.status == lib.OPD_ERR_INVALID_ARG
+    with pytest.raises(lib.OpdError) as e2:
+        ag.OPDSurrogateLoss.apply(x["H_s"], x["W_s"], tokens, lp, lp + 0.5, mask, bad_seg, n_ids, 1.0, 1e-8)
+    assert e2.value.status == lib.OPD_ERR_INVALID_ARG
+    # good ids in debug mode: no error
+    ag.score_tokens(x["H_s"], x["W_s"], tokens, mask)
